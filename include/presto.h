@@ -1,0 +1,237 @@
+/*
+ * presto.h - C ABI of the PRESTO tree draft-and-verify step on one GB300 (sm_103a).
+ *
+ * One round of tree-based diffusion speculative decoding (PRESTO: prefix-aligned
+ * scoring and priority-based tree search):
+ *
+ *   presto_topk             per-position log-softmax and top-k of the drafter logits
+ *   presto_score_build_tree prefix-aligned scores + best-first tree up to N nodes
+ *   presto_tree_mask        ancestor bitmask and position ids of the tree tokens
+ *   presto_tree_attention   tree-masked GQA attention against the KV-cache prefix
+ *   presto_accept           longest accepted root path under greedy verification
+ *
+ * Conventions shared by every call
+ *   - All array pointers are DEVICE pointers owned by the caller.  The library never
+ *     allocates, frees or synchronises; each call only enqueues work on `stream`
+ *     (a cudaStream_t; NULL is the legacy default stream) and returns.
+ *   - Arrays are dense, row-major (C order) with the shapes given below, unless a
+ *     stride argument says otherwise.
+ *   - Return value: PRESTO_OK, or a negative PRESTO_ERR_* code found on the host
+ *     before anything is enqueued (arguments, limits, workspace size), or
+ *     PRESTO_ERR_CUDA when a launch fails (cudaGetLastError).
+ *   - `dev_status` (nullable) points to one device int32.  Kernels OR PRESTO_DEV_*
+ *     bits into it when they meet bad data (an out-of-range parent or token, a
+ *     kv_len above Tmax, ...) or a bounded wait that ran out; they never trap.
+ *     The caller clears it and reads it back when it wants to check.
+ *   - Workspaces are device scratch of at least the size the matching
+ *     presto_*_workspace() query returns (256-byte aligned).  Their contents on
+ *     entry do not matter.  Two calls that run at the same time need two
+ *     workspaces.
+ *   - Limits: V < 2^18, 1 <= L <= 63, 1 <= b <= k <= 16, 1 <= N <= 256 (these let
+ *     the tree-order key pack into 64 bits), D in {64, 128}, Hq % Hkv == 0 with
+ *     Hq / Hkv a power of two <= 128.
+ *
+ * Sizes: B batch (sequences), L drafter block length (tree depth limit), V vocab,
+ * k candidates per position, b branching factor, N node budget including the root,
+ * Tmax KV-cache capacity, kv_len[b] <= Tmax committed tokens of sequence b,
+ * Hq / Hkv query / key-value heads, D head dim.
+ */
+#ifndef PRESTO_H
+#define PRESTO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* presto_stream_t;  /* same type as cudaStream_t */
+
+/* ---- host status codes ---------------------------------------------------- */
+#define PRESTO_OK 0
+#define PRESTO_ERR_INVALID_ARG (-1)   /* null pointer, bad size or dtype          */
+#define PRESTO_ERR_UNSUPPORTED (-2)   /* a documented limit is exceeded           */
+#define PRESTO_ERR_CUDA (-3)          /* a CUDA call or kernel launch failed      */
+#define PRESTO_ERR_WORKSPACE (-4)     /* workspace missing or too small           */
+
+/* ---- device status bits (ORed into *dev_status) --------------------------- */
+#define PRESTO_DEV_BAD_PARENT 0x1     /* parent index not in [0, node index)      */
+#define PRESTO_DEV_BAD_TOKEN 0x2      /* token id outside [0, V) / [0, 2^18)      */
+#define PRESTO_DEV_BAD_KVLEN 0x4      /* kv_len < 0 or kv_len > Tmax              */
+#define PRESTO_DEV_BAD_NNODES 0x8     /* n_nodes outside [1, N]                   */
+#define PRESTO_DEV_POSITIVE_SCORE 0x10 /* a token score s > 0 (log-probs must be <= 0) */
+#define PRESTO_DEV_TIMEOUT 0x20       /* a bounded in-kernel wait ran out         */
+#define PRESTO_DEV_DUP_SIBLING 0x40   /* two candidates of one position share a token */
+#define PRESTO_DEV_TABLE_FULL 0x80    /* n-gram insert found no free slot         */
+#define PRESTO_DEV_NONFINITE 0x100    /* a logits row has no finite maximum       */
+
+/* ---- element types -------------------------------------------------------- */
+#define PRESTO_F32 0
+#define PRESTO_BF16 1
+
+/* Human-readable name of a PRESTO_OK / PRESTO_ERR_* code (static string). */
+const char* presto_status_string(int status);
+
+/* ABI version: (major << 16) | minor. */
+int presto_version(void);
+
+/*
+ * presto_topk - per-row log-softmax and top-k (the drafter's position-wise
+ * marginals q_d of §2.3, Eq. marginal-surrogate; "extracts top-k diffusion
+ * candidates", §4.3; k = 10 in §5.1).
+ *
+ *   logits      [B*L rows, row_stride elements]  dtype PRESTO_F32 or PRESTO_BF16;
+ *               row r = b*L + (d-1) holds position d of sequence b; only the
+ *               first V entries of a row are read.  Values must be finite or -inf.
+ *   topk_ids    [B, L, k] int32 out: the k largest logits of each row in
+ *               descending order; equal values are ordered by lower token id.
+ *   topk_logq   [B, L, k] float32 out: log q_d(t) = x_t - log sum_v exp(x_v).
+ *   lse         [B, L] float32 out, nullable: log sum_v exp(x_v).
+ *   ws          presto_topk_workspace(B, L, V, k) bytes.
+ *   dev_status  nullable; PRESTO_DEV_NONFINITE when a row has no finite maximum.
+ * One pass over the logits; accumulation in float32.
+ */
+size_t presto_topk_workspace(int B, int L, int V, int k);
+int presto_topk(const void* logits, int dtype, int B, int L, int V, long long row_stride,
+                int k, int32_t* topk_ids, float* topk_logq, float* lse, void* ws,
+                size_t ws_bytes, int32_t* dev_status, presto_stream_t stream);
+
+/*
+ * Trigram prefix signal rho_d(t | t_{d-2}, t_{d-1}) (§4.1; the paper instantiates
+ * it with an n = 3 n-gram model, §5.1).  An open-addressing hash table in device
+ * memory with 2^log2_cap slots:
+ *   keys    [2^log2_cap] uint64, key = presto_ngram3_key(a, b, t); empty slots hold
+ *           PRESTO_NGRAM3_EMPTY.
+ *   logrho  [2^log2_cap] float32 log rho values (must be <= 0).
+ * A lookup that finds no key returns miss_logrho (<= 0).  The struct itself is a
+ * host value; its pointers are device pointers owned by the caller.
+ */
+#define PRESTO_NGRAM3_EMPTY 0xFFFFFFFFFFFFFFFFull
+typedef struct {
+  uint64_t* keys;
+  float* logrho;
+  uint32_t log2_cap;
+  float miss_logrho;
+} presto_ngram3;
+
+static inline uint64_t presto_ngram3_key(uint32_t a, uint32_t b, uint32_t t) {
+  return ((uint64_t)a << 36) | ((uint64_t)b << 18) | (uint64_t)t;
+}
+
+/* Mark every slot empty.  log2_cap in [4, 30]. */
+int presto_ngram3_clear(const presto_ngram3* table, presto_stream_t stream);
+
+/* Insert n (key, logrho) pairs (device arrays).  Keys must be unique and below
+ * 2^54; a key already present keeps one of its values.  A full table sets
+ * PRESTO_DEV_TABLE_FULL.  Keep the load factor below ~0.5 for short probes. */
+int presto_ngram3_insert(const presto_ngram3* table, const uint64_t* keys,
+                         const float* logrho, int n, int32_t* dev_status,
+                         presto_stream_t stream);
+
+/*
+ * presto_score_build_tree - prefix-aligned scoring and best-first tree search.
+ *
+ * Score (§4.1, Eq. path-score): s_{d,t}(c_d) = log q_d(t) + lambda * log rho(t |
+ * t_{d-2}, t_{d-1}), the context taken from (ctx2[b,0], ctx2[b,1], t_1, ...,
+ * t_{d-1}); computed in float32 as fl(fl(lambda * log rho) + log q).  With
+ * ngram == NULL the score is log q (marginal-only scoring, Eq.
+ * marginal-surrogate).  Path score S(child) = fl(S(parent) + s); S(root) = 0.
+ *
+ * Tree (§4.2, Alg. 2 with a node committed when it is popped): node 0 is the root
+ * (token ctx2[b,1], depth 0); a node at depth d < L has as children the top-b of
+ * the k candidates of depth d+1 ranked by (s desc, token asc); the result is the
+ * N nodes of this candidate tree that come first in the order
+ *   S desc, depth asc, token asc, parent index asc,
+ * stored in that order (so parent index < child index), which is the top-N
+ * prefix-closed set of §4.2 whenever every s <= 0.  Fewer than N nodes when the
+ * candidate tree is smaller.
+ *
+ *   topk_ids, topk_logq  [B, L, k] as written by presto_topk (row d-1 = depth d);
+ *                        tokens of one row must be distinct.
+ *   ctx2        [B, 2] int32: the last two committed tokens; ctx2[b,1] is the root.
+ *   ngram       host pointer to the table descriptor, or NULL.
+ *   lambda      >= 0 (0.2 in §5.1).
+ *   node_token  [B, N] int32 out  (-1 in unused slots)
+ *   node_parent [B, N] int32 out  (-1 for the root and unused slots)
+ *   node_depth  [B, N] int32 out  (-1 in unused slots)
+ *   node_score  [B, N] float32 out S (-inf in unused slots)
+ *   n_nodes     [B] int32 out
+ *   ws          presto_build_workspace(B, L, k, N) bytes.
+ */
+size_t presto_build_workspace(int B, int L, int k, int N);
+int presto_score_build_tree(const int32_t* topk_ids, const float* topk_logq, int B, int L,
+                            int k, int b, const int32_t* ctx2, const presto_ngram3* ngram,
+                            float lambda, int N, int32_t* node_token, int32_t* node_parent,
+                            int32_t* node_depth, float* node_score, int32_t* n_nodes,
+                            void* ws, size_t ws_bytes, int32_t* dev_status,
+                            presto_stream_t stream);
+
+/*
+ * presto_tree_mask - tree attention mask and position ids (§4.3 and App. C (I),
+ * (IV): each draft token attends to its ancestors in the draft tree).
+ *
+ *   node_parent, node_depth [B, N], n_nodes [B], kv_len [B]  int32 inputs.
+ *   mask    [B, N, ceil(N/32)] uint32 out: bit j of row i is set iff node j is node
+ *           i or one of its ancestors; rows of unused slots are 0.
+ *   pos_ids [B, N] int32 out: kv_len[b] + depth(i); -1 in unused slots.
+ */
+int presto_tree_mask(const int32_t* node_parent, const int32_t* node_depth,
+                     const int32_t* n_nodes, const int32_t* kv_len, int B, int N,
+                     uint32_t* mask, int32_t* pos_ids, int32_t* dev_status,
+                     presto_stream_t stream);
+
+/*
+ * presto_tree_attention - one layer's tree-masked GQA attention of the N tree
+ * tokens (target verification with a tree-structured mask, §5.1; App. C (I)).
+ *
+ * out[b,i,h] = sum_j softmax_j(sm_scale * <q[b,i,h], key_j>) value_j over
+ *   - the committed prefix: key_j = k_cache[b,g,j], value_j = v_cache[b,g,j],
+ *     j < kv_len[b], and
+ *   - the tree: key = k_tree[b,j,g], value = v_tree[b,j,g] for every j with bit j
+ *     of mask[b,i] set,
+ * with g = h / (Hq/Hkv).  bf16 inputs, float32 softmax and accumulation, bf16 out.
+ *
+ *   q        [B, N, Hq, D] bf16 (positions / RoPE already applied)
+ *   k_cache, v_cache [B, Hkv, Tmax, D] bf16; rows >= kv_len[b] are ignored
+ *   kv_len   [B] int32 in [0, Tmax]
+ *   k_tree, v_tree   [B, N, Hkv, D] bf16
+ *   mask     [B, N, ceil(N/32)] uint32 from presto_tree_mask
+ *   n_nodes  [B] int32; rows i >= n_nodes[b] are written as zeros (lse -inf)
+ *   out      [B, N, Hq, D] bf16 out
+ *   lse      [B, N, Hq] float32 out, nullable: natural-log softmax denominator
+ *   ws       presto_attn_workspace(B, N, Hq, Hkv, D, Tmax) bytes (for the current
+ *            device).
+ * All base pointers must be 16-byte aligned.
+ */
+size_t presto_attn_workspace(int B, int N, int Hq, int Hkv, int D, int Tmax);
+int presto_tree_attention(const void* q, const void* k_cache, const void* v_cache,
+                          const int32_t* kv_len, int Tmax, const void* k_tree,
+                          const void* v_tree, const uint32_t* mask, const int32_t* n_nodes,
+                          int B, int N, int Hq, int Hkv, int D, float sm_scale, void* out,
+                          float* lse, void* ws, size_t ws_bytes, int32_t* dev_status,
+                          presto_stream_t stream);
+
+/*
+ * presto_accept - greedy (temperature 0) verification of the tree (§2.1: tokens
+ * are accepted left to right until the first mismatch; App. A alpha_T(P); App. C
+ * (I): the position after the last accepted token takes the target's own token).
+ *
+ *   node_token, node_parent, node_depth [B, N], n_nodes [B], mask [B, N, ceil(N/32)]
+ *   target_token [B, N] int32: the target model's greedy next token after node i.
+ *   accept_len  [B] int32 out: depth of the deepest node whose every ancestor-or-self
+ *               j != 0 has node_token[j] == target_token[parent(j)].
+ *   accept_path [B, L+1] int32 out: node ids root..deepest, then -1.
+ *   bonus       [B] int32 out: target_token of the deepest accepted node.
+ */
+int presto_accept(const int32_t* node_token, const int32_t* node_parent,
+                  const int32_t* node_depth, const uint32_t* mask, const int32_t* n_nodes,
+                  const int32_t* target_token, int B, int N, int L, int32_t* accept_len,
+                  int32_t* accept_path, int32_t* bonus, int32_t* dev_status,
+                  presto_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PRESTO_H */

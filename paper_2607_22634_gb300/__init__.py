@@ -1,0 +1,26 @@
+"""PRESTO tree draft-and-verify step on one GB300 (sm_103a).
+
+The computation lives in libpresto.so (hand-written CUDA, C ABI in
+include/presto.h); this package holds its build script, a ctypes binding with the
+same entry-point names, and `DraftVerifyStep`, which keeps one round's buffers
+resident and replays the five calls (optionally as one CUDA graph).
+"""
+
+from ._lib import (  # noqa: F401
+    DEV_STATUS_BITS,
+    Ngram3Table,
+    PrestoError,
+    dev_status_names,
+    lib_path,
+    load,
+    pack_trigram_keys,
+    presto_accept,
+    presto_attn_workspace,
+    presto_build_workspace,
+    presto_score_build_tree,
+    presto_topk,
+    presto_topk_workspace,
+    presto_tree_attention,
+    presto_tree_mask,
+)
+from .step import DraftVerifyStep  # noqa: F401

@@ -1,0 +1,108 @@
+"""One round of the draft-and-verify hot path with resident buffers.
+
+`DraftVerifyStep` owns every intermediate and workspace of a round for fixed
+shapes, so a round is five library calls with no allocation:
+
+    presto_topk -> presto_score_build_tree -> presto_tree_mask
+      -> presto_tree_attention (x layers) -> presto_accept
+
+and can be captured once into a CUDA graph and replayed.
+"""
+
+from __future__ import annotations
+
+import torch
+
+from . import _lib as P
+
+
+class DraftVerifyStep:
+    def __init__(self, B, L, V, k, N, Hq, Hkv, D, Tmax, logits_dtype=torch.bfloat16,
+                 b=None, lam=0.2, ngram=None, device="cuda"):
+        self.B, self.L, self.V, self.k, self.N = B, L, V, k, N
+        self.Hq, self.Hkv, self.D, self.Tmax = Hq, Hkv, D, Tmax
+        self.b = k if b is None else b
+        self.lam = lam
+        self.ngram = ngram
+        self.device = torch.device(device)
+        i32, f32, bf = torch.int32, torch.float32, torch.bfloat16
+        dev = self.device
+        W = (N + 31) // 32
+        self.topk_ids = torch.empty(B, L, k, dtype=i32, device=dev)
+        self.topk_logq = torch.empty(B, L, k, dtype=f32, device=dev)
+        self.lse = torch.empty(B, L, dtype=f32, device=dev)
+        self.tree = {"token": torch.empty(B, N, dtype=i32, device=dev),
+                     "parent": torch.empty(B, N, dtype=i32, device=dev),
+                     "depth": torch.empty(B, N, dtype=i32, device=dev),
+                     "score": torch.empty(B, N, dtype=f32, device=dev),
+                     "n_nodes": torch.empty(B, dtype=i32, device=dev)}
+        self.mask = torch.empty(B, N, W, dtype=i32, device=dev)
+        self.pos_ids = torch.empty(B, N, dtype=i32, device=dev)
+        self.attn_out = torch.empty(B, N, Hq, D, dtype=bf, device=dev)
+        self.attn_lse = torch.empty(B, N, Hq, dtype=f32, device=dev)
+        self.accept_len = torch.empty(B, dtype=i32, device=dev)
+        self.accept_path = torch.empty(B, L + 1, dtype=i32, device=dev)
+        self.bonus = torch.empty(B, dtype=i32, device=dev)
+        self.dev_status = torch.zeros(1, dtype=i32, device=dev)
+        u8 = torch.uint8
+        self.ws_topk = torch.empty(max(P.presto_topk_workspace(B, L, V, k), 1), dtype=u8, device=dev)
+        self.ws_build = torch.empty(max(P.presto_build_workspace(B, L, k, N), 1), dtype=u8, device=dev)
+        self.ws_attn = torch.empty(max(P.presto_attn_workspace(B, N, Hq, Hkv, D, Tmax), 1),
+                                   dtype=u8, device=dev)
+        self.graph = None
+
+    CALLS = ("topk", "build", "mask", "attention", "accept")
+
+    def run(self, logits, ctx2, layers, kv_len, target_token, stream=None, marks=None):
+        """One round.  `layers` is a list of dicts with q, k_cache, v_cache, k_tree,
+        v_tree (one per attention layer).  Results stay in the step's buffers.
+        `marks` (optional) maps a call name to a (start, end) pair of CUDA events
+        recorded around that call on the launch stream."""
+        s = torch.cuda.current_stream(self.device) if stream is None else stream
+
+        def mark(name, i):
+            if marks is not None and name in marks:
+                marks[name][i].record(s)
+
+        mark("topk", 0)
+        P.presto_topk(logits, self.k, self.topk_ids, self.topk_logq, self.lse, ws=self.ws_topk,
+                      dev_status=self.dev_status, stream=s)
+        mark("topk", 1)
+        mark("build", 0)
+        P.presto_score_build_tree(self.topk_ids, self.topk_logq, ctx2, self.ngram, self.lam,
+                                  self.N, b=self.b, out=self.tree, ws=self.ws_build,
+                                  dev_status=self.dev_status, stream=s)
+        mark("build", 1)
+        mark("mask", 0)
+        P.presto_tree_mask(self.tree["parent"], self.tree["depth"], self.tree["n_nodes"], kv_len,
+                           self.mask, self.pos_ids, dev_status=self.dev_status, stream=s)
+        mark("mask", 1)
+        mark("attention", 0)
+        for lay in layers:
+            P.presto_tree_attention(lay["q"], lay["k_cache"], lay["v_cache"], kv_len,
+                                    lay["k_tree"], lay["v_tree"], self.mask,
+                                    self.tree["n_nodes"], out=self.attn_out, lse=self.attn_lse,
+                                    ws=self.ws_attn, dev_status=self.dev_status, stream=s)
+        mark("attention", 1)
+        mark("accept", 0)
+        P.presto_accept(self.tree["token"], self.tree["parent"], self.tree["depth"], self.mask,
+                        self.tree["n_nodes"], target_token, self.L, self.accept_len,
+                        self.accept_path, self.bonus, dev_status=self.dev_status, stream=s)
+        mark("accept", 1)
+
+    def kernels_per_round(self, n_layers=1):
+        """Library kernels one round launches (the split-KV combine adds one per layer)."""
+        splits = self.ws_attn.numel() > 256
+        return 4 + n_layers * (2 if splits else 1)
+
+    def capture(self, logits, ctx2, layers, kv_len, target_token):
+        """Capture one round on these exact input tensors into a CUDA graph."""
+        s = torch.cuda.Stream(device=self.device)
+        s.wait_stream(torch.cuda.current_stream(self.device))
+        with torch.cuda.stream(s):
+            self.run(logits, ctx2, layers, kv_len, target_token, stream=s)  # warm, outside graph
+        torch.cuda.current_stream(self.device).wait_stream(s)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            self.run(logits, ctx2, layers, kv_len, target_token, stream=s)
+        return g

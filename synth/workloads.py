@@ -75,7 +75,7 @@ WORKLOADS = {
     # 1 x 8 x 4096 fp32 logits, k=4, N=16; 4 q-heads / 1 kv-head, D=64, T=256.
     "tiny": Workload("tiny", B=1, L=8, V=4096, k=4, N=16, lam=0.2, use_table=True,
                      logits="planted", logits_dtype="f32", Hq=4, Hkv=1, D=64,
-                     T=256, T_min=256, seed=0, table_log2_cap=16,
+                     T=256, T_min=256, seed=0, table_log2_cap=19,
                      n_background=20_000, sigma_z=1.0),
     # Qwen3-8B-shaped dedicated-drafter round: B=1, L=16, k=8, N=64, GQA 32/8,
     # D=128, T=4096.

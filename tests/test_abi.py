@@ -1,0 +1,96 @@
+"""The C-ABI library builds, loads and exports every entry point that
+include/presto.h declares; host-side validation rejects bad arguments before any
+work is enqueued.  No kernel runs here (CPU only)."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2607_22634_gb300 as P
+from paper_2607_22634_gb300 import _lib
+
+HDR = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "presto.h")
+
+
+def declared_functions():
+    src = open(HDR).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    names = re.findall(r"^\s*(?:const\s+)?[A-Za-z_][\w\s\*]*?\b(presto_\w+)\s*\(", src, flags=re.M)
+    inline = set(re.findall(r"static\s+inline\s+\w+\s+(presto_\w+)", src))
+    return sorted(set(names) - inline)
+
+
+def test_header_declares_the_five_steps():
+    names = declared_functions()
+    for n in ("presto_topk", "presto_score_build_tree", "presto_tree_mask",
+              "presto_tree_attention", "presto_accept"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol():
+    lib = ctypes.CDLL(P.load() and _lib.lib_path())
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+    # and the binding declares a signature for each of them
+    assert set(declared_functions()) <= set(_lib._SIGS)
+
+
+def test_version_and_status_strings():
+    lib = P.load()
+    assert lib.presto_version() >> 16 == 1
+    for code in (0, -1, -2, -3, -4):
+        assert lib.presto_status_string(code).startswith(b"PRESTO")
+
+
+N = None
+
+
+def test_host_validation_rejects_bad_arguments():
+    lib = P.load()
+    p = ctypes.c_void_p(16)  # never dereferenced: every call below fails validation first
+    # null logits
+    assert lib.presto_topk(N, 1, 1, 1, 10, 10, 2, p, p, N, N, 0, N, N) == -1
+    # bad dtype
+    assert lib.presto_topk(p, 7, 1, 1, 10, 10, 2, p, p, N, N, 0, N, N) == -1
+    # k > V
+    assert lib.presto_topk(p, 1, 1, 1, 4, 4, 5, p, p, N, N, 0, N, N) == -1
+    # k above the packing limit
+    assert lib.presto_topk(p, 1, 1, 1, 100, 100, 17, p, p, N, N, 0, N, N) == -2
+    # V beyond 2^18
+    assert lib.presto_topk(p, 1, 1, 1, 1 << 18, 1 << 18, 4, p, p, N, N, 0, N, N) == -2
+    # row stride below V
+    assert lib.presto_topk(p, 1, 1, 1, 100, 99, 4, p, p, N, N, 0, N, N) == -1
+    # build: b > k, N > 256, negative lambda
+    args = lambda B, L, k, b, lam, Nn: (p, p, B, L, k, b, p, None, ctypes.c_float(lam), Nn,
+                                        p, p, p, p, p, N, 0, N, N)
+    assert lib.presto_score_build_tree(*args(1, 4, 4, 5, 0.2, 8)) == -1
+    assert lib.presto_score_build_tree(*args(1, 4, 4, 4, 0.2, 257)) == -2
+    assert lib.presto_score_build_tree(*args(1, 4, 4, 4, -0.5, 8)) == -1
+    assert lib.presto_score_build_tree(*args(1, 64, 4, 4, 0.2, 8)) == -2
+    # mask: N beyond limit
+    assert lib.presto_tree_mask(p, p, p, p, 1, 300, p, p, N, N) == -2
+    # attention: head dim, GQA ratio, misalignment
+    att = lambda D, Hq, Hkv, q=p: (q, p, p, p, 64, p, p, p, p, 1, 8, Hq, Hkv, D,
+                                   ctypes.c_float(0.1), p, N, N, 0, N, N)
+    assert lib.presto_tree_attention(*att(96, 8, 2)) == -2
+    assert lib.presto_tree_attention(*att(128, 12, 4)) == -2      # G = 3 not a power of two
+    assert lib.presto_tree_attention(*att(128, 8, 3)) == -1       # Hq % Hkv != 0
+    assert lib.presto_tree_attention(*att(128, 8, 2, q=ctypes.c_void_p(24))) == -1
+    # accept: L above limit
+    assert lib.presto_accept(p, p, p, p, p, p, 1, 8, 64, p, p, p, N, N) == -2
+    # table: capacity out of range
+    bad = _lib.Ngram3(16, 16, 40, -12.0)
+    assert lib.presto_ngram3_clear(ctypes.byref(bad), N) == -1
+
+
+def test_binding_raises_on_error_status():
+    with pytest.raises(_lib.PrestoError):
+        _lib._check(-2, "x")
+
+
+def test_trigram_key_packing():
+    k = _lib.pack_trigram_keys([1, 262143], [2, 0], [3, 262143])
+    assert int(k[0]) == (1 << 36) | (2 << 18) | 3
+    assert int(k[1]) == (262143 << 36) | 262143

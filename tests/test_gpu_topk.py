@@ -1,0 +1,78 @@
+"""presto_topk (GPU, through the C ABI) vs the oracle: ids bit-exact, log q and
+lse within 1e-5 * max(1, |x|)."""
+
+import numpy as np
+import pytest
+import torch
+
+import synth
+import paper_2607_22634_gb300 as P
+from oracle import presto_oracle as O
+from gpu_common import GPU, rel_close
+
+pytestmark = GPU
+
+
+def _check(logits_cpu, k, view=None):
+    """logits_cpu: [B, L, V] CPU tensor; view(t) may return a strided view on device."""
+    B, L, V = logits_cpu.shape
+    dev = logits_cpu.cuda()
+    if view is not None:
+        dev = view(dev)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ids, logq, lse = P.presto_topk(dev, k, dev_status=st)
+    torch.cuda.synchronize()
+    oids, ologq, olse = O.topk_logsoftmax(logits_cpu.reshape(B * L, V).double().numpy(), k)
+    np.testing.assert_array_equal(ids.cpu().numpy().reshape(B * L, k), oids)
+    assert rel_close(logq.cpu().numpy().reshape(B * L, k), ologq) <= 1e-5
+    assert rel_close(lse.cpu().numpy().reshape(-1), olse) <= 1e-5
+    return int(st.item())
+
+
+@pytest.mark.parametrize("name", ["tiny", "qwen3_8b", "self_spec", "long_ctx", "batched_ragged"])
+def test_topk_workloads(name):
+    w = synth.WORKLOADS[name]
+    x = synth.drafter_logits(w)
+    assert _check(x, w.k) == 0
+
+
+@pytest.mark.parametrize("V,dtype,k", [(4097, torch.float32, 4), (1001, torch.bfloat16, 7),
+                                       (16, torch.float32, 16), (31, torch.bfloat16, 1),
+                                       (151936, torch.bfloat16, 16), (8, torch.bfloat16, 8),
+                                       (70000, torch.float32, 10)])
+def test_topk_ragged_vocab_and_k(V, dtype, k):
+    g = torch.Generator().manual_seed(V + k)
+    x = (torch.randn(3, 5, V, generator=g) * 3).to(dtype)
+    assert _check(x, k) == 0
+
+
+def test_topk_unaligned_rows_use_plain_loads():
+    g = torch.Generator().manual_seed(7)
+    for dtype in (torch.float32, torch.bfloat16):
+        wide = (torch.randn(2, 6, 5003, generator=g) * 2).to(dtype)
+        V = 4999
+        sub = wide[:, :, :V].contiguous()       # the oracle sees the same values
+        assert _check(sub, 6, view=lambda t, w=wide: w.cuda()[:, :, :V]) == 0
+
+
+def test_topk_many_ties_and_masked_vocab():
+    g = torch.Generator().manual_seed(3)
+    x = torch.round(torch.randn(2, 8, 20000, generator=g) * 2) / 2   # values on a 0.5 grid
+    x[:, :, ::3] = -float("inf")                                       # masked tokens
+    assert _check(x.to(torch.bfloat16), 9) == 0
+    assert _check(x, 16) == 0
+
+
+def test_topk_large_magnitudes():
+    g = torch.Generator().manual_seed(4)
+    x = torch.randn(1, 4, 30000, generator=g) * 40
+    assert _check(x, 5) == 0
+
+
+def test_topk_all_masked_row_reports_nonfinite():
+    x = torch.full((1, 2, 300), -float("inf"))
+    x[0, 1, 5] = 1.0
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    P.presto_topk(x.cuda(), 2, dev_status=st)
+    torch.cuda.synchronize()
+    assert int(st.item()) & 0x100

@@ -98,6 +98,27 @@ int presto_topk(const void* logits, int dtype, int B, int L, int V, long long ro
                 size_t ws_bytes, int32_t* dev_status, presto_stream_t stream);
 
 /*
+ * presto_topk_noalloc - presto_topk for callers that cannot allocate device memory.
+ * The paper has no counterpart; this is a deployment variant of presto_topk.
+ *
+ * Same arguments and results as presto_topk, without the workspace: the span
+ * partials live in a file-scope device array of PRESTO_TOPK_STATIC_SCRATCH_BYTES
+ * (1 MiB) that every GPU loading this library keeps for the life of the process.
+ * Returns PRESTO_ERR_UNSUPPORTED, enqueueing nothing, when
+ * presto_topk_workspace(B, L, V, k) exceeds that size.  Calls no cudaMalloc or
+ * cudaFree.  The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current) and caches it; make that
+ * first call before any stream capture.  All calls on a device share the one
+ * array, so calls whose kernels may overlap on the GPU race; order them on one
+ * stream.  The array keeps the last call's contents; the call clears what must
+ * start at zero on `stream` itself.
+ */
+#define PRESTO_TOPK_STATIC_SCRATCH_BYTES (1u << 20)
+int presto_topk_noalloc(const void* logits, int dtype, int B, int L, int V,
+                        long long row_stride, int k, int32_t* topk_ids, float* topk_logq,
+                        float* lse, int32_t* dev_status, presto_stream_t stream);
+
+/*
  * Trigram prefix signal rho_d(t | t_{d-2}, t_{d-1}) (§4.1; the paper instantiates
  * it with an n = 3 n-gram model, §5.1).  An open-addressing hash table in device
  * memory with 2^log2_cap slots:

@@ -47,6 +47,7 @@ _SIGS = {
     "presto_topk_workspace": (ctypes.c_size_t, [_I, _I, _I, _I]),
     "presto_topk": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, _P, _P, _P, _P,
                          ctypes.c_size_t, _P, _P]),
+    "presto_topk_noalloc": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, _P, _P, _P, _P, _P]),
     "presto_ngram3_clear": (_I, [ctypes.POINTER(Ngram3), _P]),
     "presto_ngram3_insert": (_I, [ctypes.POINTER(Ngram3), _P, _P, _I, _P, _P]),
     "presto_build_workspace": (ctypes.c_size_t, [_I, _I, _I, _I]),
@@ -148,6 +149,24 @@ def presto_topk(logits, k, topk_ids=None, topk_logq=None, lse=None, ws=None, dev
                             _ptr(topk_logq), _ptr(lse), _ptr(ws), nws, _ptr(dev_status),
                             _stream(stream))
     _check(st, "presto_topk")
+    return topk_ids, topk_logq, lse
+
+
+def presto_topk_noalloc(logits, k, topk_ids, topk_logq, lse=None, dev_status=None, stream=None):
+    """presto_topk without a workspace: for callers that must not allocate device
+    memory.  The library keeps the scratch in a fixed 1 MiB device array shared
+    by every call on the device, so calls that may overlap on the GPU race.
+    Outputs must be passed in (nothing is allocated here either)."""
+    B, L, V = logits.shape
+    dtype = {torch.float32: PRESTO_F32, torch.bfloat16: PRESTO_BF16}.get(logits.dtype)
+    if dtype is None or logits.stride(2) != 1:
+        raise ValueError("logits must be float32 or bfloat16 with unit last stride")
+    _need(topk_ids, torch.int32, (B, L, k), "topk_ids")
+    _need(topk_logq, torch.float32, (B, L, k), "topk_logq")
+    st = load().presto_topk_noalloc(_ptr(logits), dtype, B, L, V, logits.stride(1), k,
+                                    _ptr(topk_ids), _ptr(topk_logq), _ptr(lse), _ptr(dev_status),
+                                    _stream(stream))
+    _check(st, "presto_topk_noalloc")
     return topk_ids, topk_logq, lse
 
 

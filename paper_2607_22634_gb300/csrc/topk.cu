@@ -12,6 +12,8 @@
 //     merge in the CTA that finishes last (atomic ticket), which writes the row.
 #include <cuda_bf16.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 namespace presto {
@@ -473,4 +475,65 @@ extern "C" int presto_topk(const void* logits, int dtype, int B, int L, int V,
   else
     topk_kernel<__nv_bfloat16><<<grid, kThreads, smem, stream>>>(a);
   return launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free top-k.
+//
+// Some callers cannot hand this library a workspace: a plugin running inside an
+// inference server whose device memory all belongs to the host framework's
+// allocator, a C caller with no allocator handle at all, or a latency-critical
+// loop that must not call cudaMalloc (which can block on device-wide
+// synchronisation and fail under fragmentation).  For them this entry point
+// keeps the span partials of presto_topk in a fixed file-scope device array
+// instead of a caller workspace, and otherwise runs the same code.
+//
+// The array costs kStaticScratchBytes on every GPU that loads this library, for
+// the life of the process.  All calls on one device share it: two calls whose
+// kernels overlap on the GPU (different streams, no ordering between them) race
+// on it.  Its contents persist between calls; the per-row tickets that must
+// start at zero are cleared by an async memset on the caller's stream at every
+// call, and everything else is written before it is read.
+// ---------------------------------------------------------------------------
+namespace presto {
+namespace {
+
+constexpr size_t kStaticScratchBytes = PRESTO_TOPK_STATIC_SCRATCH_BYTES;
+__device__ __align__(256) unsigned char g_topk_scratch[kStaticScratchBytes];
+
+std::mutex g_scratch_mutex;
+void* g_scratch_addr[64] = {};
+
+// Device address of g_topk_scratch for the current device.  Host code cannot use
+// the symbol itself (its host-side name is only a stand-in), so the address is
+// looked up once per device, with that device current, and cached.
+void* static_scratch() {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_topk_scratch) != cudaSuccess || !p) return nullptr;
+    g_scratch_addr[dev] = p;
+  }
+  return g_scratch_addr[dev];
+}
+
+}  // namespace
+}  // namespace presto
+
+extern "C" int presto_topk_noalloc(const void* logits, int dtype, int B, int L, int V,
+                                   long long row_stride, int k, int32_t* topk_ids,
+                                   float* topk_logq, float* lse, int32_t* dev_status,
+                                   presto_stream_t stream) {
+  PRESTO_CHECK_ARG(logits && topk_ids && topk_logq);
+  PRESTO_CHECK_ARG(dtype == PRESTO_F32 || dtype == PRESTO_BF16);
+  PRESTO_CHECK_ARG(B >= 1 && L >= 1 && V >= 1 && k >= 1 && k <= V && row_stride >= V);
+  PRESTO_CHECK_LIMIT(k <= kMaxK && V < kMaxV && L <= kMaxL);
+  const size_t need = presto_topk_workspace(B, L, V, k);
+  if (need > kStaticScratchBytes) return PRESTO_ERR_UNSUPPORTED;
+  void* ws = static_scratch();
+  if (!ws) return PRESTO_ERR_CUDA;
+  return presto_topk(logits, dtype, B, L, V, row_stride, k, topk_ids, topk_logq, lse, ws,
+                     kStaticScratchBytes, dev_status, stream);
 }

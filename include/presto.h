@@ -103,7 +103,7 @@ int presto_topk(const void* logits, int dtype, int B, int L, int V, long long ro
  *
  * Same arguments and results as presto_topk, without the workspace: the span
  * partials live in a file-scope device array of PRESTO_TOPK_STATIC_SCRATCH_BYTES
- * (1 MiB) that every GPU loading this library keeps for the life of the process.
+ * (16 KiB) that every GPU loading this library keeps for the life of the process.
  * Returns PRESTO_ERR_UNSUPPORTED, enqueueing nothing, when
  * presto_topk_workspace(B, L, V, k) exceeds that size.  Calls no cudaMalloc or
  * cudaFree.  The first call on a device looks up the array's device address
@@ -113,7 +113,7 @@ int presto_topk(const void* logits, int dtype, int B, int L, int V, long long ro
  * stream.  The array keeps the last call's contents; the call clears what must
  * start at zero on `stream` itself.
  */
-#define PRESTO_TOPK_STATIC_SCRATCH_BYTES (1u << 20)
+#define PRESTO_TOPK_STATIC_SCRATCH_BYTES (1u << 14)
 int presto_topk_noalloc(const void* logits, int dtype, int B, int L, int V,
                         long long row_stride, int k, int32_t* topk_ids, float* topk_logq,
                         float* lse, int32_t* dev_status, presto_stream_t stream);

@@ -154,7 +154,7 @@ def presto_topk(logits, k, topk_ids=None, topk_logq=None, lse=None, ws=None, dev
 
 def presto_topk_noalloc(logits, k, topk_ids, topk_logq, lse=None, dev_status=None, stream=None):
     """presto_topk without a workspace: for callers that must not allocate device
-    memory.  The library keeps the scratch in a fixed 1 MiB device array shared
+    memory.  The library keeps the scratch in a fixed 16 KiB device array shared
     by every call on the device, so calls that may overlap on the GPU race.
     Outputs must be passed in (nothing is allocated here either)."""
     B, L, V = logits.shape

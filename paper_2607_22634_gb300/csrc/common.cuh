@@ -31,7 +31,7 @@ inline int launch_status() {
   return cudaGetLastError() == cudaSuccess ? PRESTO_OK : PRESTO_ERR_CUDA;
 }
 
-inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+__host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Per-device SM count, cached (host).
 int sm_count();

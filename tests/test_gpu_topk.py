@@ -36,6 +36,15 @@ def test_topk_workloads(name):
     assert _check(x, w.k) == 0
 
 
+def test_topk_few_rows_spread_over_many_ctas():
+    """A handful of long rows: each row spans more CTAs than one cluster holds and
+    the spans merge through the workspace."""
+    g = torch.Generator().manual_seed(11)
+    for B, L in ((1, 1), (1, 4), (2, 3)):
+        x = (torch.randn(B, L, 151936, generator=g) * 2).to(torch.bfloat16)
+        assert _check(x, 10) == 0
+
+
 @pytest.mark.parametrize("V,dtype,k", [(4097, torch.float32, 4), (1001, torch.bfloat16, 7),
                                        (16, torch.float32, 16), (31, torch.bfloat16, 1),
                                        (151936, torch.bfloat16, 16), (8, torch.bfloat16, 8),

@@ -37,10 +37,13 @@ def _noalloc(lib, x, k):
     return rc, ids, logq, lse, int(st.item())
 
 
-@pytest.mark.parametrize("name", ["tiny", "qwen3_8b", "self_spec"])
+@pytest.mark.parametrize("name", ["tiny", "qwen3_8b", "self_spec", "qwen3_8b_4rows"])
 def test_noalloc_topk_matches_workspace_entry_point(name):
     lib = P.load()
-    w = synth.WORKLOADS[name]
+    if name == "qwen3_8b_4rows":   # few long rows: the shape whose spans merge in scratch
+        w = synth.WORKLOADS["qwen3_8b"].scaled(L=4)
+    else:
+        w = synth.WORKLOADS[name]
     x = synth.drafter_logits(w).cuda()
     ref_ids, ref_logq, ref_lse = P.presto_topk(x, w.k)
     torch.cuda.synchronize()
@@ -54,10 +57,11 @@ def test_noalloc_topk_matches_workspace_entry_point(name):
 
 def test_noalloc_rejects_shapes_beyond_its_scratch():
     lib = P.load()
-    # 16384 rows x k = 16 needs more span scratch than the fixed array holds
-    B, L, V, k = 512, 32, 1000, 16
-    assert P.presto_topk_workspace(B, L, V, k) > (1 << 20)
-    x = torch.zeros(B, L, V, dtype=torch.bfloat16, device="cuda")
+    # nine rows of a near-2^18 float32 vocabulary with k = 16 spread each row over
+    # ~22 CTAs whose partial lists need more scratch than the fixed array holds
+    B, L, V, k = 1, 9, 262143, 16
+    assert P.presto_topk_workspace(B, L, V, k) > (1 << 14)
+    x = torch.zeros(B, L, V, dtype=torch.float32, device="cuda")
     rc, ids, _, _, _ = _noalloc(lib, x, k)
     assert rc == -2                          # PRESTO_ERR_UNSUPPORTED, nothing enqueued
     assert int(ids.min()) == -7 and int(ids.max()) == -7

@@ -7,15 +7,16 @@
 //     the candidate tree and computes, for every candidate j of depth d+1 under
 //     that context, s = log q + lambda log rho (hash-table probes, batched so their
 //     loads overlap), keeps the top-b by (s desc, token asc) as 8-byte records that
-//     already hold the child's key bits, and notes whether fp32 rounding can reorder
-//     two kept siblings; it writes them into the leader CTA's shared memory
-//     (distributed shared memory), then the cluster synchronises once.
-//   phase 2 (leader, warp 0): the pop loop.  A frontier entry carries a 64-bit key packing
-//     the total order (S desc, depth asc, token asc, parent index asc), so two
-//     warp-wide max reductions find the next node.  Each committed node owns one
-//     entry (its next child not yet taken), held in a fixed register slot of a fixed
-//     lane: popping a child advances its parent's entry to the next sibling and
-//     gives the new node an entry for its first child (lazy sibling enumeration).
+//     already hold the child's key bits, and writes them into the leader CTA's
+//     shared memory (distributed shared memory); the cluster then synchronises once.
+//   phase 2 (leader CTA): the nodes the best-first loop commits are the N - 1
+//     largest keys of the candidate tree (key = S desc, depth asc, token asc, parent
+//     index asc, packed into 64 bits), because a child's key is always below its
+//     parent's.  They are found level by level with the whole CTA: the N - 1
+//     largest keys among nodes of depth <= d are kept sorted; the children of the
+//     newest level that beat the smallest kept key are ranked against them.  L
+//     block-wide steps replace N - 1 dependent pops, with the same nodes in the
+//     same order.
 #include <cooperative_groups.h>
 
 #include <initializer_list>
@@ -101,46 +102,37 @@ __device__ __forceinline__ uint32_t ordered(float f) {
 __device__ __forceinline__ float unordered(uint32_t o) {
   return __uint_as_float((o & 0x80000000u) ? (o & 0x7fffffffu) : ~o);
 }
-// Frontier key: larger key = earlier in the total order (S desc, depth asc, token
-// asc, parent index asc).  Zero never occurs for a real node (ordered(-inf) > 0).
-__device__ __forceinline__ uint64_t make_key(float S, int depth, int token, int parent) {
-  return (static_cast<uint64_t>(ordered(S)) << 32) |
-         (static_cast<uint64_t>(63 - depth) << 26) |
-         (static_cast<uint64_t>(0x3FFFF - token) << 8) | static_cast<uint64_t>(255 - parent);
-}
 
 struct Smem {
-  int tok[kMaxN];
-  int par[kMaxN];
-  int dep[kMaxN];
-  float S[kMaxN];
   int cid[kMaxL][kMaxK];          // candidate tokens of every depth
   float clq[kMaxL][kMaxK];        // their log q
   int ctx0, ctx1;
+  int nc;                         // candidates of the current level (phase 2)
 };
 
 // Tables of one sequence, indexed by context c = d * ctx_stride + ci (d = depth of
 // the children - 1, ci = context pair index):
-//   kid  uint2[c][b]  the top-b candidates of the context in (s desc, token asc)
-//                     order: x = bits of s, y = the key bits of (depth d+1, token)
-//                     with the candidate index in the low byte (the parent field
-//                     of the key, filled in when the child is generated)
-//   info float2[c]    (smallest gap between s-adjacent kept candidates whose tokens
-//                     are in descending order, largest |s| among them)
+//   kid  uint2[c][b]  the top-b candidates of the context by (s desc, token asc),
+//                     in no particular order: x = bits of s, y = the key bits of
+//                     (depth d+1, token) with the candidate index in the low byte
+//                     (the parent field of the key, filled in when the child is
+//                     generated)
 // With a prefix signal ctx_stride = k*k (contexts (t_{d-1}, t_d) as index pairs);
 // marginal-only scoring has one context per depth.
 struct TableLayout {
   int cs, nctx;
-  size_t info_off, bytes;
+  size_t bytes;
   __host__ __device__ TableLayout(int L, int k, int bf, int use_table) {
     cs = use_table ? k * k : 1;
     nctx = L * cs;
-    info_off = static_cast<size_t>(nctx) * bf * 8;
-    bytes = align_up(info_off + static_cast<size_t>(nctx) * 8, 16);
+    bytes = align_up(static_cast<size_t>(nctx) * bf * 8, 16);
   }
 };
-__host__ __device__ inline size_t child_bytes(int N, int bf) {
-  return align_up(static_cast<size_t>(N) * bf * 9, 16);  // uint64 keys + payload bytes
+// Child record of candidate j (token t) of depth d+1 under some context, score s.
+__device__ __forceinline__ uint2 kid_record(float s, int d, int t, int j) {
+  return make_uint2(__float_as_uint(s), (static_cast<uint32_t>(63 - (d + 1)) << 26) |
+                                            (static_cast<uint32_t>(0x3FFFF - t) << 8) |
+                                            static_cast<uint32_t>(j));
 }
 // Flat context id g (over live contexts only) -> (d, ci).
 __device__ __forceinline__ void decode_ctx(int g, int k, int use_table, int& d, int& ci) {
@@ -161,173 +153,187 @@ __device__ __forceinline__ void decode_ctx(int g, int k, int use_table, int& d, 
 }
 constexpr size_t kDynSmemBudget = 200 * 1024;
 constexpr int kCluster = 8;
-constexpr float kTieMargin = 4.8e-7f;  // 2^-21: fp32 sums closer than this may round equal
 
-// Best-first pop loop of the leader CTA's warp 0 (see file header).
-// SLOTS = frontier register slots per lane (ceil(N / 32), a power of two).
-template <int SLOTS>
-__device__ __forceinline__ int pop_loop(const Args& a, Smem& sm, const uint2* kids,
-                                        const float2* info, uint64_t* chkey,
-                                        unsigned char* chpay, int lane) {
+// Phase-2 scratch of the leader CTA (aliases the phase-1 staging area).  The kept
+// set A (non-root nodes, sorted by key, so A[r] is node r + 1) is double-buffered;
+// C holds one level's candidates.  Per entry: key, the index of its own children's
+// context (kNoCtx at depth L), its candidate index j, and its parent's node index.
+struct P2Layout {
+  size_t akey, axc, apid, aj, ckey, cxc, cpid, cj, rk, bytes;
+  __host__ __device__ P2Layout(int N, int bf) {
+    const size_t na = N, nc = static_cast<size_t>(N) * bf;
+    size_t o = 0;
+    akey = o;  o += 2 * na * 8;
+    ckey = o;  o += nc * 8;
+    axc = o;   o += 2 * na * 4;
+    cxc = o;   o += nc * 4;
+    apid = o;  o += align_up(2 * na * 2, 4);
+    cpid = o;  o += align_up(nc * 2, 4);
+    rk = o;    o += align_up((na + nc) * 2, 4);
+    aj = o;    o += align_up(2 * na, 4);
+    cj = o;    o += align_up(nc, 4);
+    bytes = align_up(o, 16);
+  }
+};
+constexpr uint32_t kNoCtx = 0xFFFFFFFFu;
+
+// Top-N selection of the candidate tree, level by level (leader CTA, all threads).
+//
+// Best-first expansion with lazy commits pops nodes in decreasing key order (a
+// child's key is below its parent's: S does not grow along a path and ties go to
+// the shallower node), so its N - 1 committed nodes are the N - 1 largest keys of
+// the whole tree.  After step d, A holds the N - 1 largest keys among nodes of
+// depth <= d.  Step d + 1 only needs the children of A's depth-d nodes: any node
+// of depth d + 1 among the N - 1 largest of depth <= d + 1 has its parent among the
+// N - 1 largest of depth <= d, and its key exceeds tau, the smallest key of a full
+// A.  The candidates that pass are ranked against A and the N - 1 largest kept.
+// A node's final index is its rank, so the parent index in the key (the last tie
+// break) is the parent's rank in A, consistent across steps.
+// Returns the node count (root included).
+__device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigned char* p2,
+                             int tid) {
   const int L = a.L, k = a.k, N = a.N, nb = a.bf;
   const int cs = a.use_table ? k * k : 1;
-  uint64_t fk[SLOTS];
-  uint32_t fp[SLOTS];
-#pragma unroll
-  for (int r = 0; r < SLOTS; ++r) {
-    fk[r] = 0ull;
-    fp[r] = 0u;
-  }
-  uint64_t best = 0ull;
-  uint32_t best_pay = 0u;
-  int best_slot = 0;
-  // lane-local maximum over the slots, as a tree of independent comparisons
-  auto rescan = [&]() {
-    uint64_t kb[SLOTS];
-    uint32_t pb[SLOTS];
-    int sb[SLOTS];
-#pragma unroll
-    for (int r = 0; r < SLOTS; ++r) {
-      kb[r] = fk[r];
-      pb[r] = fp[r];
-      sb[r] = r;
-    }
-#pragma unroll
-    for (int w = 1; w < SLOTS; w *= 2)
-#pragma unroll
-      for (int r = 0; r + w < SLOTS; r += 2 * w)
-        if (kb[r + w] > kb[r]) {
-          kb[r] = kb[r + w];
-          pb[r] = pb[r + w];
-          sb[r] = sb[r + w];
-        }
-    best = kb[0];
-    best_pay = pb[0];
-    best_slot = sb[0];
-  };
-  auto set_slot = [&](int slot, uint64_t key, uint32_t pay) {
-#pragma unroll
-    for (int r = 0; r < SLOTS; ++r)
-      if (r == slot) {
-        fk[r] = key;
-        fp[r] = pay;
-      }
-  };
-  // Children of committed node n (depth d, score Sn, context ci of its children,
-  // own candidate index jn): the kept candidates of depth d+1 in s order, stored by
-  // key order (S desc, token asc) as n's child list.  Every lane gets the first
-  // child's key and payload (child order | candidate index << 8 | jn << 16).
-  auto expand = [&](int n, int d, float Sn, int ci, int jn, uint64_t& key0, uint32_t& pay0) {
-    key0 = 0ull;
-    pay0 = 0u;
-    if (d >= L) return;
-    const int c = d * cs + ci;
-    const bool on = lane < nb;
-    const uint2 kd = on ? kids[c * nb + lane] : make_uint2(0u, 0u);
-    const float2 inf = info[c];
-    const int j = static_cast<int>(kd.y & 0xFFu);
-    const uint64_t key = on ? (static_cast<uint64_t>(ordered(__fadd_rn(Sn, __uint_as_float(kd.x))))
-                               << 32) | (kd.y & ~0xFFu) | static_cast<uint32_t>(255 - n)
-                            : 0ull;
-    // In s order the fp32 path scores are non-increasing; siblings can leave key
-    // order only if two of them round to the same S.  `safe` rules that out.
-    const bool safe = inf.x > kTieMargin * (fabsf(Sn) + inf.y);
-    int pos = lane, src = 0;
-    if (!safe) {  // rank by key; equal keys (duplicate tokens) by lane
-      pos = 0;
-      for (int i = 0; i < nb; ++i) {
-        const uint64_t ki = __shfl_sync(kFull, key, i);
-        pos += ki > key || (ki == key && i < lane);
-      }
-      src = __ffs(__ballot_sync(kFull, on && pos == 0)) - 1;
-    }
-    if (on) {
-      chkey[n * nb + pos] = key;
-      chpay[n * nb + pos] = static_cast<unsigned char>(j);
-    }
-    key0 = __shfl_sync(kFull, key, src);
-    pay0 = (static_cast<uint32_t>(__shfl_sync(kFull, j, src)) << 8) |
-           (static_cast<uint32_t>(jn) << 16);
-  };
+  const int cap = N - 1;  // non-root nodes
+  const P2Layout ly(N, nb);
+  // A buffer b of each field starts at b * N
+  uint64_t* const akey = reinterpret_cast<uint64_t*>(p2 + ly.akey);
+  uint32_t* const axc = reinterpret_cast<uint32_t*>(p2 + ly.axc);
+  int16_t* const apid = reinterpret_cast<int16_t*>(p2 + ly.apid);
+  uint8_t* const aj = p2 + ly.aj;
+  uint64_t* ckey = reinterpret_cast<uint64_t*>(p2 + ly.ckey);
+  uint32_t* cxc = reinterpret_cast<uint32_t*>(p2 + ly.cxc);
+  int16_t* cpid = reinterpret_cast<int16_t*>(p2 + ly.cpid);
+  uint8_t* cj = p2 + ly.cj;
+  int16_t* rk = reinterpret_cast<int16_t*>(p2 + ly.rk);
 
-  if (lane == 0) {
-    sm.tok[0] = sm.ctx1;
-    sm.par[0] = -1;
-    sm.dep[0] = 0;
-    sm.S[0] = 0.f;
-  }
-  {
-    uint64_t k0;
-    uint32_t p0;
-    expand(0, 0, 0.f, 0, 0, k0, p0);
-    if (lane == 0) {
-      set_slot(0, k0, p0);
-      rescan();
+  if (tid == 0) sm.nc = 0;
+  __syncthreads();
+  int na = 0, cur = 0;
+  uint64_t tau = 0ull;  // candidates need key > tau (0: A not yet full)
+  for (int d = 0; d < L && cap > 0; ++d) {
+    // ---- candidates of depth d + 1: children of the root (d = 0) or of A's
+    // depth-d nodes
+    const int parents = d == 0 ? 1 : na;
+    for (int q = tid; q < parents * nb; q += kThreads) {
+      const int e = q / nb, c = q - e * nb;
+      uint32_t x;
+      float Sp;
+      int pnode, pj;
+      if (d == 0) {
+        x = 0u;
+        Sp = 0.f;
+        pnode = 0;
+        pj = 0;
+      } else {
+        const uint64_t ke = akey[cur * N + e];
+        if (63 - static_cast<int>((ke >> 26) & 63u) != d) continue;
+        x = axc[cur * N + e];
+        if (x == kNoCtx) continue;
+        Sp = unordered(static_cast<uint32_t>(ke >> 32));
+        pnode = e + 1;
+        pj = aj[cur * N + e];
+      }
+      const uint2 kd = kids[x * nb + c];
+      const uint64_t key =
+          (static_cast<uint64_t>(ordered(__fadd_rn(Sp, __uint_as_float(kd.x)))) << 32) |
+          (kd.y & ~0xFFu) | static_cast<uint32_t>(255 - pnode);
+      if (key <= tau) continue;
+      const int jc = static_cast<int>(kd.y & 0xFFu);
+      const int dc = d + 1;
+      const uint32_t xc = dc >= L ? kNoCtx
+                                  : static_cast<uint32_t>(
+                                        dc * cs + (!a.use_table ? 0 : (dc == 1 ? jc : pj * k + jc)));
+      const int slot = atomicAdd(&sm.nc, 1);
+      ckey[slot] = key;
+      cxc[slot] = xc;
+      cpid[slot] = static_cast<int16_t>(pnode);
+      cj[slot] = static_cast<uint8_t>(jc);
     }
+    __syncthreads();
+    const int m = sm.nc;
+    if (m == 0) break;  // no node of depth d + 1 can be kept: none deeper either
+    // ---- ranks in A u C by (key desc, position asc); A is sorted
+    const int ne = na + m;
+    for (int e = tid; e < ne; e += kThreads) {
+      int r;
+      if (e < na) {
+        const uint64_t ke = akey[cur * N + e];
+        r = e;
+        for (int i = 0; i < m; ++i) r += ckey[i] > ke;
+      } else {
+        const int ci = e - na;
+        const uint64_t ke = ckey[ci];
+        int lo = 0, hi = na;  // A entries with key >= ke
+        while (lo < hi) {
+          const int mid = (lo + hi) >> 1;
+          if (akey[cur * N + mid] >= ke) lo = mid + 1;
+          else hi = mid;
+        }
+        r = lo;
+        for (int i = 0; i < m; ++i) {
+          const uint64_t ki = ckey[i];
+          r += ki > ke || (ki == ke && i < ci);
+        }
+      }
+      rk[e] = static_cast<int16_t>(r < cap ? r : cap);
+    }
+    __syncthreads();
+    // ---- the cap largest become the new A; parent indices follow their ranks
+    const int nxt = cur ^ 1;
+    for (int e = tid; e < ne; e += kThreads) {
+      const int r = rk[e];
+      if (r >= cap) continue;
+      int pid;
+      if (e < na) {
+        akey[nxt * N + r] = akey[cur * N + e];
+        axc[nxt * N + r] = axc[cur * N + e];
+        aj[nxt * N + r] = aj[cur * N + e];
+        pid = apid[cur * N + e];
+      } else {
+        akey[nxt * N + r] = ckey[e - na];
+        axc[nxt * N + r] = cxc[e - na];
+        aj[nxt * N + r] = cj[e - na];
+        pid = cpid[e - na];
+      }
+      if (pid > 0) {
+        const int pr = rk[pid - 1];
+        if (pr >= cap || pr >= r) report(a.dev_status, PRESTO_DEV_BAD_PARENT);  // s > 0 input
+        pid = pr < cap ? pr + 1 : 0;
+      }
+      apid[nxt * N + r] = static_cast<int16_t>(pid);
+    }
+    if (tid == 0) sm.nc = 0;  // every thread read it before the last barrier
+    na = ne < cap ? ne : cap;
+    cur = nxt;
+    __syncthreads();
+    if (na == cap) tau = akey[cur * N + cap - 1];
   }
-  __syncwarp();
-  int n = 1;
-  while (n < N) {
-    const unsigned hi = static_cast<unsigned>(best >> 32), lo = static_cast<unsigned>(best);
-    const unsigned mh = __reduce_max_sync(kFull, hi);
-    if (mh == 0u) break;  // frontier empty
-    const unsigned cand = __ballot_sync(kFull, hi == mh);
-    int win;
-    unsigned ml;
-    if ((cand & (cand - 1u)) == 0u) {  // one lane holds the largest S (common case)
-      win = __ffs(cand) - 1;
-      ml = __shfl_sync(kFull, lo, win);
+  // ---- write the tree: node 0 is the root, node r + 1 is A[r]
+  for (int i = tid; i < N; i += kThreads) {
+    const size_t o = static_cast<size_t>(blockIdx.x / kCluster) * N + i;
+    if (i == 0) {
+      a.node_token[o] = sm.ctx1;
+      a.node_parent[o] = -1;
+      a.node_depth[o] = 0;
+      a.node_score[o] = 0.f;
+    } else if (i <= na) {
+      const uint64_t ke = akey[cur * N + i - 1];
+      const uint32_t lo = static_cast<uint32_t>(ke);
+      a.node_token[o] = 0x3FFFF - static_cast<int>((lo >> 8) & 0x3FFFFu);
+      a.node_depth[o] = 63 - static_cast<int>((lo >> 26) & 63u);
+      a.node_parent[o] = apid[cur * N + i - 1];
+      a.node_score[o] = unordered(static_cast<uint32_t>(ke >> 32));
     } else {
-      ml = __reduce_max_sync(kFull, hi == mh ? lo : 0u);
-      win = __ffs(__ballot_sync(kFull, hi == mh && lo == ml)) - 1;
+      a.node_token[o] = -1;
+      a.node_parent[o] = -1;
+      a.node_depth[o] = -1;
+      a.node_score[o] = -INFINITY;
     }
-    const uint32_t pay = __shfl_sync(kFull, best_pay, win);
-    const float S = unordered(mh);
-    const int d = 63 - static_cast<int>((ml >> 26) & 63u);
-    const int t = 0x3FFFF - static_cast<int>((ml >> 8) & 0x3FFFFu);
-    const int p = 255 - static_cast<int>(ml & 255u);
-    const int c = static_cast<int>(pay & 0xFFu);
-    const int j = static_cast<int>((pay >> 8) & 0xFFu);
-    const int jp = static_cast<int>((pay >> 16) & 0xFFu);
-    if (p >= n || d < 1 || d > L || j >= k || c >= nb) {  // cannot happen on valid input
-      if (lane == 0) report(a.dev_status, PRESTO_DEV_BAD_PARENT);
-      break;
-    }
-    // p's next child (every parent of a frontier entry has b children; the loads
-    // are issued now and used after the expansion below)
-    const int c2 = c + 1;
-    const bool more = c2 < nb;
-    const uint64_t nk = more ? chkey[p * nb + c2] : 0ull;
-    const uint32_t np = more ? static_cast<uint32_t>(c2) |
-                                   (static_cast<uint32_t>(chpay[p * nb + c2]) << 8) |
-                                   (static_cast<uint32_t>(jp) << 16)
-                             : 0u;
-    if (lane == 0) {
-      sm.tok[n] = t;
-      sm.par[n] = p;
-      sm.dep[n] = d;
-      sm.S[n] = S;
-    }
-    // children of n see the context (t_{d-1}, t_d)
-    const int ci = !a.use_table ? 0 : (d == 1 ? j : jp * k + j);
-    uint64_t k0;
-    uint32_t p0;
-    expand(n, d, S, ci, j, k0, p0);
-    // frontier update: p's entry moves on to its next child (lane win), n gets an
-    // entry for its first child (lane n % 32)
-    const bool upd_win = lane == win, upd_own = lane == (n & 31) && k0 != 0ull;
-    if (upd_win || upd_own) {
-      if (upd_win) set_slot(best_slot, nk, np);
-      if (upd_own) set_slot(n >> 5, k0, p0);
-      rescan();
-    }
-    ++n;
-    __syncwarp();  // node arrays and child lists written above are read later
   }
-  return n;
+  return na + 1;
 }
 
-template <int SLOTS>
 __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   namespace cg = cooperative_groups;
   extern __shared__ __align__(16) unsigned char dyn[];
@@ -339,18 +345,15 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   const int L = a.L, k = a.k, N = a.N, nb = a.bf, use_table = a.use_table;
   const TableLayout tl(L, k, nb, use_table);
   // leader's tables: in its shared memory (seen through DSMEM) or in the workspace
-  const size_t cb = child_bytes(N, nb);
   unsigned char* tables;
   if (a.tables_in_smem)
-    tables = static_cast<unsigned char*>(cluster.map_shared_rank(static_cast<void*>(dyn + cb), 0));
+    tables = static_cast<unsigned char*>(cluster.map_shared_rank(static_cast<void*>(dyn), 0));
   else
     tables = a.g_tables + static_cast<size_t>(b) * tl.bytes;
   uint2* kids = reinterpret_cast<uint2*>(tables);
-  float2* info = reinterpret_cast<float2*>(tables + tl.info_off);
   // this CTA's staging area: scores and order of its share of the contexts
-  const size_t stage_off = cb + (a.tables_in_smem ? tl.bytes : 0);
+  const size_t stage_off = a.tables_in_smem ? tl.bytes : 0;
   float* st_s = reinterpret_cast<float*>(dyn + stage_off);
-  unsigned char* st_o = dyn + stage_off + static_cast<size_t>(a.per_cta) * k * 4;
 
   // ---- candidates and context
   for (int i = tid; i < L * k; i += kThreads) {
@@ -437,81 +440,46 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
         sc = __fadd_rn(__fmul_rn(a.lambda, lr), lq[q]);
       }
       if (sc > 0.f) report(a.dev_status, PRESTO_DEV_POSITIVE_SCORE);
-      st_s[f] = sc;
-    }
-  }
-  __syncthreads();
-  // rank of each candidate within its context, strict total order (float bits as
-  // integers, then token, then index) so ranks form a permutation even for
-  // duplicate tokens or NaN
-  for (int f = tid; f < my; f += kThreads) {
-    const int gl = f / k, j = f - gl * k;
-    int d, ci;
-    decode_ctx(g0 + gl, k, use_table, d, ci);
-    const float* row = st_s + gl * k;
-    const uint32_t sj = ordered(row[j]);
-    const int tj = sm.cid[d][j];
-    int rk = 0;
-    for (int i = 0; i < k; ++i) {
-      const uint32_t si = ordered(row[i]);
-      const int ti = sm.cid[d][i];
-      rk += (si > sj) || (si == sj && (ti < tj || (ti == tj && i < j)));
-    }
-    st_o[gl * k + rk] = static_cast<unsigned char>(j);
-  }
-  __syncthreads();
-  // kept children of every context, in s order, into the leader's tables
-  for (int f = tid; f < (g1 - g0) * nb; f += kThreads) {
-    const int gl = f / nb, r = f - gl * nb;
-    int d, ci;
-    decode_ctx(g0 + gl, k, use_table, d, ci);
-    const int j = st_o[gl * k + r];
-    const uint32_t lowbits = (static_cast<uint32_t>(63 - (d + 1)) << 26) |
-                             (static_cast<uint32_t>(0x3FFFF - sm.cid[d][j]) << 8) |
-                             static_cast<uint32_t>(j);
-    kids[(d * tl.cs + ci) * nb + r] = make_uint2(__float_as_uint(st_s[gl * k + j]), lowbits);
-  }
-  // per context: can fp32 rounding reorder two kept siblings?
-  for (int gl = tid; gl < g1 - g0; gl += kThreads) {
-    int d, ci;
-    decode_ctx(g0 + gl, k, use_table, d, ci);
-    float gap = INFINITY, mag = 0.f;
-    for (int r = 0; r < nb; ++r) {
-      const int jr = st_o[gl * k + r];
-      const float sr = st_s[gl * k + jr];
-      mag = fmaxf(mag, fabsf(sr));
-      if (r + 1 < nb) {
-        const int jn = st_o[gl * k + r + 1];
-        if (sm.cid[d][jr] > sm.cid[d][jn]) gap = fminf(gap, sr - st_s[gl * k + jn]);
+      if (nb == k) {  // every candidate is kept
+        const int gl = f / k, j = f - gl * k;
+        int d, ci;
+        decode_ctx(g0 + gl, k, use_table, d, ci);
+        kids[(d * tl.cs + ci) * nb + j] = kid_record(sc, d, sm.cid[d][j], j);
+      } else {
+        st_s[f] = sc;
       }
     }
-    if (!(mag < INFINITY)) gap = 0.f;  // non-finite scores: always rank by key
-    info[d * tl.cs + ci] = make_float2(gap, mag);
+  }
+  __syncthreads();
+  // with b < k: keep the top-b of every context by a strict total order (float
+  // bits as integers, then token, then index; a permutation even for duplicate
+  // tokens or NaN)
+  if (nb < k) {
+    __syncthreads();
+    for (int f = tid; f < my; f += kThreads) {
+      const int gl = f / k, j = f - gl * k;
+      int d, ci;
+      decode_ctx(g0 + gl, k, use_table, d, ci);
+      const float* row = st_s + gl * k;
+      const uint32_t sj = ordered(row[j]);
+      const int tj = sm.cid[d][j];
+      int rk = 0;
+      for (int i = 0; i < k; ++i) {
+        const uint32_t si = ordered(row[i]);
+        const int ti = sm.cid[d][i];
+        rk += (si > sj) || (si == sj && (ti < tj || (ti == tj && i < j)));
+      }
+      if (rk < nb) kids[(d * tl.cs + ci) * nb + rk] = kid_record(row[j], d, sm.cid[d][j], j);
+    }
   }
   if (!a.tables_in_smem) __threadfence();
   cluster.sync();  // the leader's tables are complete
-  if (rank != 0 || tid >= 32) return;
+  if (rank != 0) return;
 
-  // ---- phase 2: best-first pop loop (leader, warp 0)
-  uint64_t* chkey = reinterpret_cast<uint64_t*>(dyn);
-  unsigned char* chpay = dyn + static_cast<size_t>(N) * nb * 8;
-  int n;
-  if (a.tables_in_smem)  // separate instance so the table loads are shared-memory loads
-    n = pop_loop<SLOTS>(a, sm, reinterpret_cast<const uint2*>(dyn + cb),
-                        reinterpret_cast<const float2*>(dyn + cb + tl.info_off), chkey, chpay,
-                        lane);
-  else
-    n = pop_loop<SLOTS>(a, sm, kids, info, chkey, chpay, lane);
-  // ---- write the tree
-  for (int i = lane; i < N; i += 32) {
-    const size_t o = static_cast<size_t>(b) * N + i;
-    const bool used = i < n;
-    a.node_token[o] = used ? sm.tok[i] : -1;
-    a.node_parent[o] = used ? sm.par[i] : -1;
-    a.node_depth[o] = used ? sm.dep[i] : -1;
-    a.node_score[o] = used ? sm.S[i] : -INFINITY;
-  }
-  if (lane == 0) a.n_nodes[b] = n;
+  // ---- phase 2: top-N selection, level by level (leader CTA)
+  const int n = select_levels(a, sm, a.tables_in_smem ? reinterpret_cast<const uint2*>(dyn) : kids,
+                              dyn + stage_off, tid);
+  if (tid == 0) a.n_nodes[b] = n;
 }
 
 }  // namespace
@@ -543,7 +511,12 @@ extern "C" int presto_ngram3_insert(const presto_ngram3* t, const uint64_t* keys
 }
 
 namespace {
-size_t stage_bytes(int per_cta, int k) { return align_up(static_cast<size_t>(per_cta) * k * 5, 16); }
+// phase-1 staging area of each CTA, reused by the leader for phase 2
+size_t stage_bytes(int per_cta, int k, int N, int bf) {
+  const size_t st = align_up(static_cast<size_t>(per_cta) * k * 4, 16);
+  const size_t p2 = P2Layout(N, bf).bytes;
+  return st > p2 ? st : p2;
+}
 int contexts_all(int L, int k, int use_table) {
   if (!use_table) return L;
   return 1 + (L > 1 ? k : 0) + (L > 2 ? (L - 2) * k * k : 0);
@@ -556,7 +529,7 @@ extern "C" size_t presto_build_workspace(int B, int L, int k, int N) {
   // live here (sized for the prefix-signal case, the larger one).
   const TableLayout tl(L, k, k, 1);
   const int per = (contexts_all(L, k, 1) + kCluster - 1) / kCluster;
-  const size_t smem = child_bytes(N, k) + tl.bytes + stage_bytes(per, k);
+  const size_t smem = tl.bytes + stage_bytes(per, k, N, k);
   return smem <= kDynSmemBudget ? 256 : align_up(B * tl.bytes, 256);
 }
 
@@ -596,8 +569,8 @@ extern "C" int presto_score_build_tree(const int32_t* topk_ids, const float* top
   a.nctx_all = contexts_all(L, k, a.use_table);
   a.per_cta = (a.nctx_all + kCluster - 1) / kCluster;
   const TableLayout tl(L, k, b, a.use_table);
-  const size_t cb = child_bytes(N, b), sb = stage_bytes(a.per_cta, k);
-  a.tables_in_smem = cb + tl.bytes + sb <= kDynSmemBudget;
+  const size_t sb = stage_bytes(a.per_cta, k, N, b);
+  a.tables_in_smem = tl.bytes + sb <= kDynSmemBudget;
   if (!a.tables_in_smem) {
     if (!ws || reinterpret_cast<uintptr_t>(ws) % 16 || ws_bytes < static_cast<size_t>(B) * tl.bytes)
       return PRESTO_ERR_WORKSPACE;
@@ -609,16 +582,11 @@ extern "C" int presto_score_build_tree(const int32_t* topk_ids, const float* top
   a.node_score = node_score;
   a.n_nodes = n_nodes;
   a.dev_status = dev_status;
-  const size_t smem = cb + (a.tables_in_smem ? tl.bytes : 0) + sb;
+  const size_t smem = (a.tables_in_smem ? tl.bytes : 0) + sb;
   if (smem > kDynSmemBudget) return PRESTO_ERR_UNSUPPORTED;
-  void (*kernel)(Args);
-  const int slots = (N + 31) / 32;
-  kernel = slots <= 1 ? build_kernel<1> : slots <= 2 ? build_kernel<2>
-         : slots <= 4 ? build_kernel<4> : build_kernel<8>;
   static bool attr_set = [] {
-    for (auto fn : {build_kernel<1>, build_kernel<2>, build_kernel<4>, build_kernel<8>})
-      cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           static_cast<int>(kDynSmemBudget));
+    cudaFuncSetAttribute(build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         static_cast<int>(kDynSmemBudget));
     return true;
   }();
   (void)attr_set;
@@ -634,6 +602,6 @@ extern "C" int presto_score_build_tree(const int32_t* topk_ids, const float* top
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (cudaLaunchKernelEx(&cfg, kernel, a) != cudaSuccess) return PRESTO_ERR_CUDA;
+  if (cudaLaunchKernelEx(&cfg, build_kernel, a) != cudaSuccess) return PRESTO_ERR_CUDA;
   return launch_status();
 }

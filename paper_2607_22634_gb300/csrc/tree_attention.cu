@@ -6,24 +6,24 @@
 // dense contraction against that head's keys, so it runs on the 5th-generation
 // tensor cores, ping-ponging two 128-row tiles per CTA:
 //   * one CTA per (sequence, kv head, pair of 128-row tiles, KV split);
-//   * warp 16 issues TMA loads (both Q tiles once, then one K and one V tile of 128
-//     keys at a time; K is refilled as soon as both QK^T products have read it, V as
-//     soon as both PV products have);
-//   * warp 17 issues tcgen05.mma into TMEM: S_t = Q_t K^T (128 fp32 columns per
-//     tile) and O_t += P_t V (D columns per tile), interleaved so that the tensor
-//     core works on one tile while the other tile's softmax runs;
-//   * warps 0-7 and 8-15 run the softmax of tiles 0 and 1, two threads per query
-//     row (TMEM lane), each on 64 of the 128 key columns: tcgen05.ld of S,
-//     prefix-length and ancestor-bitmask masks, online softmax (the two halves of a
-//     row exchange their maxima through shared memory), P (bf16, 128-byte swizzled
-//     K-major) to shared memory.
-//     The running maximum is only moved (and O rescaled in TMEM) when it grows by
-//     more than 2^8, so most tiles skip the rescale;
+//   * warp 8 loads both Q tiles, then K tiles of 64 keys into a 4-deep ring; warp 10
+//     loads V tiles into a 3-deep ring (TMA, 128-byte swizzle).  A K slot is refilled
+//     once both QK^T products of its tile completed, a V slot once both PV products
+//     did;
+//   * warp 9 issues tcgen05.mma: S_t = Q_t K^T (64 fp32 TMEM columns per row tile) one
+//     KV tile ahead of O_t += P_t V, where P_t (bf16) is read from TMEM.  The whole
+//     warp runs the issue loop and one elected lane issues, so descriptors stay on the
+//     uniform datapath;
+//   * warps 0-3 and 4-7 run the softmax of tiles 0 and 1, one thread per query row
+//     (TMEM lane): tcgen05.ld of S, prefix-length and ancestor-bitmask masks (full
+//     prefix tiles skip them), online softmax with packed fp32x2 arithmetic, and
+//     tcgen05.st of P.  The running maximum is only moved (and O rescaled in TMEM)
+//     when it grows by more than 2^8, so most tiles skip the rescale;
 //   * with several KV splits, the splits of one row block form a thread-block
-//     cluster: each CTA leaves its fp32 O and (m, l) per row in its own shared
-//     memory, the cluster synchronises, and each CTA merges a slice of the rows
-//     from all peers through distributed shared memory (log-sum-exp weighting)
-//     and writes them; no partials go to global memory.
+//     cluster (up to 16 CTAs): each CTA writes its rows' (m, l) and unnormalised fp32
+//     O to the workspace (column-quad-major, coalesced), the cluster synchronises
+//     (release / acquire), and each CTA merges a slice of the rows over the splits
+//     with log-sum-exp weights, all loads of a row issued together.
 // Every wait is bounded; on time-out the CTA records PRESTO_DEV_TIMEOUT and unwinds.
 #include <cuda_bf16.h>
 
@@ -40,24 +40,26 @@ namespace presto {
 namespace {
 
 constexpr int kBM = 128;        // query rows per tile (TMEM lanes)
-constexpr int kBN = 128;        // keys per tile
-// 18 warps: per row tile 8 softmax warps (two threads per query row, each taking 64
-// of the 128 key columns), then the TMA warp and the MMA warp
-constexpr int kSoftWarps = 8;
-constexpr int kThreads = (2 * kSoftWarps + 2) * 32;
-constexpr int kTmaWarp = 2 * kSoftWarps;
-constexpr int kMmaWarp = 2 * kSoftWarps + 1;
-constexpr int kSoftThreads = kSoftWarps * 32;  // per tile
+constexpr int kBN = 64;         // keys per KV tile
+constexpr int kKStages = 4;     // K ring depth (K is needed two tiles before V)
+constexpr int kVStages = 3;     // V ring depth
+// 11 warps: 0-3 and 4-7 run the softmax of row tiles 0 and 1 (one thread per query
+// row = TMEM lane), 8 loads Q and K, 9 issues tensor-core MMAs, 10 loads V
+constexpr int kThreads = 352;
+constexpr int kKWarp = 8;
+constexpr int kMmaWarp = 9;
+constexpr int kVWarp = 10;
+constexpr int kSoftThreads = 128;  // per tile
 constexpr float kRescaleLog2 = 8.f;  // move the running max only when it grows by > 2^8
-constexpr int kPanelBytes = 128 * 128;  // 128 rows x 128 bytes (64 bf16)
+constexpr int kRowBytes = 128;       // one 128-byte-swizzled row: 64 bf16
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
-constexpr uint32_t kTmemCols = 512;  // S0 | S1 | O0 | O1, 128 columns each
-// fp32 partial O rows left in shared memory for the cluster merge: padded so that
-// a warp's 16-byte stores to 32 consecutive rows spread over the banks
-template <int D>
-constexpr int kPartStride = D + 4;
-constexpr int kMaxSplits = 8;  // KV splits of a row block = CTAs of its (portable) cluster
+// TMEM columns: S of tile t (64 fp32) at 64t, P of tile t (64 bf16 packed in pairs)
+// at 128 + 32t, O of tile t at 256 + 128t
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kTmemP = 128;
+constexpr uint32_t kTmemO = 256;
+constexpr int kMaxSplits = 16;  // KV splits of a row block = CTAs of its cluster
 
 struct Args {
   const int32_t* kv_len;
@@ -67,124 +69,72 @@ struct Args {
   float scale_log2;
   __nv_bfloat16* out;
   float* lse;
+  float4* part_o;   // KV splits: unnormalised fp32 O [CTA][D / 4][2 * kBM] (column quads)
+  float2* part_ml;  // KV splits: (m, l) per row [CTA][2 * kBM], log2 domain
   int32_t* dev_status;
 };
 
+// Shared memory: Q of both row tiles, the K ring, the V ring.  Every operand is
+// stored as 64-column panels of 128-byte rows with the 128-byte swizzle (Q: 128 rows
+// per panel, K and V: 64 rows per panel).
 template <int D>
 struct Layout {
   static constexpr int kPanels = D / 64;
+  static constexpr int kQPanel = kBM * kRowBytes;   // 16 KB
+  static constexpr int kKVPanel = kBN * kRowBytes;  // 8 KB
   static constexpr int kQBytes = kBM * D * 2;
-  static constexpr int kTileBytes = kBN * D * 2;
-  static constexpr int kPBytes = kBM * kBN * 2;
-  static constexpr int kQ = 0;                       // Q of tile 0, then tile 1
+  static constexpr int kTileBytes = kBN * D * 2;    // one K or V tile
+  static constexpr int kQ = 0;                          // tile 0, then tile 1
   static constexpr int kK = kQ + 2 * kQBytes;
-  static constexpr int kV = kK + kTileBytes;
-  static constexpr int kP = kV + kTileBytes;         // P of tile 0, then tile 1
-  static constexpr int kBytes = kP + 2 * kPBytes;
+  static constexpr int kV = kK + kKStages * kTileBytes;
+  static constexpr int kBytes = kV + kVStages * kTileBytes;
   static constexpr int kAlloc = kBytes + 1024;  // room to align the base to 1024
 };
 
 struct Bars {
   uint64_t q_full;
-  uint64_t k_full, k_empty;
-  uint64_t v_full, v_empty;
+  uint64_t k_full[kKStages], k_empty[kKStages];
+  uint64_t v_full[kVStages], v_empty[kVStages];
   uint64_t s_full[2], s_free[2];
   uint64_t p_full[2], o_done[2];
 };
 
-// Merge the KV splits of one row block (the CTAs of this cluster).  Every CTA holds
-// the fp32 partial O (unnormalised) and (m, l) of its split for the block's rows in
-// shared memory; CTA c of n merges rows [c*R/n, (c+1)*R/n) from all peers through
-// distributed shared memory and writes the bf16 output and lse.  Phases: gather the
-// peers' (m, l) of the slice, form per-row weights, then sum the peers' rows with
-// all remote loads of an item issued together.
-// Named barrier over `nthreads` threads that also returns the AND of `pred` over them.
-__device__ __forceinline__ bool bar_and(int id, int nthreads, bool pred) {
-  uint32_t r;
-  asm volatile(
-      "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n"
-      " bar.red.and.pred q, %2, %3, p;\n selp.u32 %0, 1, 0, q;\n}\n"
-      : "=r"(r)
-      : "r"(static_cast<uint32_t>(pred)), "r"(id), "r"(nthreads)
-      : "memory");
-  return r != 0;
+// Packed fp32 pairs (f32x2 arithmetic issues one instruction per two values) and
+// the three-input max.
+__device__ __forceinline__ uint64_t pack2(float x, float y) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(x), "f"(y));
+  return r;
+}
+__device__ __forceinline__ void unpack2(uint64_t r, float& x, float& y) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(x), "=f"(y) : "l"(r));
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
 }
 
-template <int D>
-__device__ void cluster_merge(const Args& a, int b, int g, int mt0, int ntiles, int nn,
-                              uint8_t* smem, float2 (*part_ml)[kBM]) {
-  namespace cg = cooperative_groups;
-  cg::cluster_group cluster = cg::this_cluster();
-  cluster.sync();  // every split's partial is in place
-  const int nsp = static_cast<int>(cluster.num_blocks());
-  const int me = static_cast<int>(cluster.block_rank());
-  const int R = ntiles * kBM;
-  const int r0 = me * R / nsp, r1 = (me + 1) * R / nsp, nr = r1 - r0;
-  constexpr int kC4 = D / 4;  // float4 columns per row
-  const int nodes_per_tile = kBM / a.G;
-  // scratch after this CTA's own partial rows (the slice has <= kBM rows):
-  // m then weight [row][split], l [row][split], 1/L [row], lse [row]
-  float* wgt = reinterpret_cast<float*>(smem) + 2 * kBM * kPartStride<D>;
-  float* lval = wgt + kBM * kMaxSplits;
-  float* rinv = lval + kBM * kMaxSplits;
-  float* rlse = rinv + kBM;
-  for (int i = threadIdx.x; i < nr * nsp; i += kThreads) {
-    const int row = r0 + i / nsp, s = i % nsp;
-    const float2 ml = *cluster.map_shared_rank(&part_ml[row / kBM][row % kBM], s);
-    wgt[(i / nsp) * kMaxSplits + s] = ml.x;
-    lval[(i / nsp) * kMaxSplits + s] = ml.y;
-  }
-  __syncthreads();
-  for (int i = threadIdx.x; i < nr; i += kThreads) {
-    float* w = wgt + i * kMaxSplits;
-    const float* lv = lval + i * kMaxSplits;
-    float M = -INFINITY;
-    for (int s = 0; s < nsp; ++s) M = fmaxf(M, w[s]);
-    float L = 0.f;
-    for (int s = 0; s < nsp; ++s) {
-      const float ws = (M == -INFINITY || w[s] == -INFINITY) ? 0.f : ex2(w[s] - M);
-      w[s] = ws;
-      L += lv[s] * ws;
-    }
-    const int row = r0 + i;
-    const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
-    const bool used = node < nn && L > 0.f;
-    rinv[i] = used ? 1.f / L : 0.f;
-    rlse[i] = used ? (M + log2f(L)) * kLn2 : -INFINITY;
-  }
-  __syncthreads();
-  for (int item = threadIdx.x; item < nr * kC4; item += kThreads) {
-    const int i = item / kC4, c4 = item % kC4;
-    const int rr = r0 + i;
-    const int t = rr / kBM, r = rr % kBM;
-    const int node = (mt0 + t) * nodes_per_tile + r / a.G, hh = r % a.G;
-    if (node >= a.N) continue;
-    const float* prow = reinterpret_cast<const float*>(smem) + rr * kPartStride<D> + c4 * 4;
-    float4 o[kMaxSplits];
+// One row's 64 scores of a KV tile -> the tile's row maximum (raw scores), as
+// eight independent three-input-max chains.
+__device__ __forceinline__ float row_max64(const float* v) {
+  float q[8];
 #pragma unroll
-    for (int s = 0; s < kMaxSplits; ++s)
-      if (s < nsp) o[s] = *reinterpret_cast<const float4*>(cluster.map_shared_rank(prow, s));
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-    for (int s = 0; s < kMaxSplits; ++s)
-      if (s < nsp) {
-        const float ws = wgt[i * kMaxSplits + s];
-        acc.x += ws * o[s].x;
-        acc.y += ws * o[s].y;
-        acc.z += ws * o[s].z;
-        acc.w += ws * o[s].w;
-      }
-    const float inv = rinv[i];
-    const size_t orow = ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
-    const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-    const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
-    uint2 u;
-    u.x = *reinterpret_cast<const uint32_t*>(&lo);
-    u.y = *reinterpret_cast<const uint32_t*>(&hi);
-    *reinterpret_cast<uint2*>(a.out + orow + c4 * 4) = u;
-    if (c4 == 0 && a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = rlse[i];
+  for (int i = 0; i < 8; ++i) {
+    const float* w = v + 8 * i;
+    q[i] = fmaxf(max3(max3(max3(w[0], w[1], w[2]), w[3], w[4]), w[5], w[6]), w[7]);
   }
-  cluster.sync();  // peers have finished reading this CTA's shared memory
+  return max3(max3(q[0], q[1], q[2]), max3(q[3], q[4], q[5]), fmaxf(q[6], q[7]));
 }
 
 template <int D>
@@ -192,6 +142,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
                 const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ CUtensorMap tm_kt,
                 const __grid_constant__ CUtensorMap tm_vt, const Args a) {
+  namespace cg = cooperative_groups;
   using Ly = Layout<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -211,49 +162,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int mt0 = mp * a.tpc;       // first row tile of the group
   const bool has1 = a.tpc == 2 && mt0 + 1 < a.n_mt;  // second tile present
   const int ntiles = has1 ? 2 : 1;
-
-  int kv = a.kv_len[b];
-  if (kv < 0 || kv > a.Tmax) {
-    if (tid == 0) report(a.dev_status, PRESTO_DEV_BAD_KVLEN);
-    kv = kv < 0 ? 0 : a.Tmax;
-  }
-  int nn = a.n_nodes[b];
-  if (nn < 0 || nn > a.N) nn = nn < 0 ? 0 : a.N;
-  const int prefix_tiles = (kv + kBN - 1) / kBN;
-  const int per = (prefix_tiles + a.n_splits - 1) / a.n_splits;
-  const int t_begin = min(split * per, prefix_tiles);
-  const int n_prefix = min(prefix_tiles, t_begin + per) - t_begin;
-  const int n_tree = split == a.n_splits - 1 ? (nn + kBN - 1) / kBN : 0;
-  const int nt = n_prefix + n_tree;
-  const int nodes_per_tile = kBM / a.G;
-
-  __shared__ float2 part_ml[2][kBM];  // (m, l) per row of this CTA's split, log2 domain
-  __shared__ float xchg[2][2][2][kBM];  // [iteration & 1][tile][half][row] row maxima
-  __shared__ float lsum[2][2][kBM];     // [tile][half][row] row sums
   const bool clustered = a.n_splits > 1;
-  if (nt == 0) {  // nothing to attend to in this split (CTA-uniform)
-    if (tid < ntiles * kBM) {
-      const int t = tid / kBM, r = tid % kBM;
-      const int node = (mt0 + t) * nodes_per_tile + r / a.G, hh = r % a.G;
-      if (clustered) {
-        part_ml[t][r] = make_float2(-INFINITY, 0.f);
-      } else if (node < a.N) {  // no keys at all: a zero row, lse -inf
-        __nv_bfloat16* orow =
-            a.out + ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
-        for (int c = 0; c < D; c += 8) *reinterpret_cast<uint4*>(orow + c) = make_uint4(0, 0, 0, 0);
-        if (a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = -INFINITY;
-      }
-    }
-    if (clustered) cluster_merge<D>(a, b, g, mt0, ntiles, nn, smem, part_ml);
-    return;
-  }
+  const int nodes_per_tile = kBM / a.G;
+  // the sequence's lengths: loaded now, used after the set-up below
+  const int kv_raw = a.kv_len[b];
+  const int nn_raw = a.n_nodes[b];
 
   if (tid == 0) {
     mbar_init(&bars.q_full, 1);
-    mbar_init(&bars.k_full, 1);
-    mbar_init(&bars.k_empty, 1);
-    mbar_init(&bars.v_full, 1);
-    mbar_init(&bars.v_empty, 1);
+    for (int st = 0; st < kKStages; ++st) {
+      mbar_init(&bars.k_full[st], 1);
+      mbar_init(&bars.k_empty[st], 1);
+    }
+    for (int st = 0; st < kVStages; ++st) {
+      mbar_init(&bars.v_full[st], 1);
+      mbar_init(&bars.v_empty[st], 1);
+    }
     for (int t = 0; t < 2; ++t) {
       mbar_init(&bars.s_full[t], 1);
       mbar_init(&bars.s_free[t], kSoftThreads);
@@ -270,129 +194,143 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+
+  int kv = kv_raw;
+  if (kv < 0 || kv > a.Tmax) {
+    if (tid == 0) report(a.dev_status, PRESTO_DEV_BAD_KVLEN);
+    kv = kv < 0 ? 0 : a.Tmax;
+  }
+  const int nn = nn_raw < 0 ? 0 : (nn_raw > a.N ? a.N : nn_raw);
+  const int prefix_tiles = (kv + kBN - 1) / kBN;
+  const int per = (prefix_tiles + a.n_splits - 1) / a.n_splits;
+  const int t_begin = min(split * per, prefix_tiles);
+  const int n_prefix = min(prefix_tiles, t_begin + per) - t_begin;
+  const int n_tree = split == a.n_splits - 1 ? (nn + kBN - 1) / kBN : 0;
+  const int nt = n_prefix + n_tree;  // KV tiles of this split (CTA-uniform)
+
   volatile int* abort = &abort_flag;
   auto fail = [&]() {
     *abort = 1;
     report(a.dev_status, PRESTO_DEV_TIMEOUT);
   };
 
-  if (warp == kTmaWarp) {
-    // ------------------------------------------------------------ TMA producer
+  if (nt > 0 && warp == kKWarp) {
+    // ------------------------------------------------------------ Q and K loads
     if (lane == 0) {
       prefetch_tensormap(&tm_q);
       prefetch_tensormap(&tm_kc);
-      prefetch_tensormap(&tm_vc);
       prefetch_tensormap(&tm_kt);
-      prefetch_tensormap(&tm_vt);
       mbar_arrive_expect_tx(&bars.q_full, ntiles * Ly::kQBytes);
       for (int t = 0; t < ntiles; ++t)
         for (int p = 0; p < Ly::kPanels; ++p)
-          tma_load_3d(smem + Ly::kQ + t * Ly::kQBytes + p * kPanelBytes, &tm_q, p * 64, g * a.G,
+          tma_load_3d(smem + Ly::kQ + t * Ly::kQBytes + p * Ly::kQPanel, &tm_q, p * 64, g * a.G,
                       b * a.N + (mt0 + t) * nodes_per_tile, &bars.q_full);
-      auto load_kv = [&](int j, bool is_v) {
-        uint64_t* bar = is_v ? &bars.v_full : &bars.k_full;
-        uint8_t* dst = smem + (is_v ? Ly::kV : Ly::kK);
-        mbar_arrive_expect_tx(bar, Ly::kTileBytes);
+      // K_j -> slot j % kKStages, once both QK^T of K_{j - kKStages} completed
+      for (int j = 0; j < nt; ++j) {
+        const int st = j % kKStages;
+        if (j >= kKStages && !mbar_wait(&bars.k_empty[st], (j / kKStages - 1) & 1, abort)) {
+          fail();
+          break;
+        }
+        uint8_t* dst = smem + Ly::kK + st * Ly::kTileBytes;
+        mbar_arrive_expect_tx(&bars.k_full[st], Ly::kTileBytes);
         for (int p = 0; p < Ly::kPanels; ++p) {
           if (j < n_prefix)
-            tma_load_3d(dst + p * kPanelBytes, is_v ? &tm_vc : &tm_kc, p * 64,
-                        (t_begin + j) * kBN, b * a.Hkv + g, bar);
+            tma_load_3d(dst + p * Ly::kKVPanel, &tm_kc, p * 64, (t_begin + j) * kBN,
+                        b * a.Hkv + g, &bars.k_full[st]);
           else
-            tma_load_3d(dst + p * kPanelBytes, is_v ? &tm_vt : &tm_kt, p * 64, g,
-                        b * a.N + (j - n_prefix) * kBN, bar);
+            tma_load_3d(dst + p * Ly::kKVPanel, &tm_kt, p * 64, g,
+                        b * a.N + (j - n_prefix) * kBN, &bars.k_full[st]);
         }
-      };
-      for (int j = 0; j < nt; ++j) {
-        if (j > 0 && !mbar_wait(&bars.k_empty, (j - 1) & 1, abort)) {
-          fail();
-          break;
-        }
-        load_kv(j, false);
-        if (j > 0 && !mbar_wait(&bars.v_empty, (j - 1) & 1, abort)) {
-          fail();
-          break;
-        }
-        load_kv(j, true);
       }
     }
-  } else if (warp == kMmaWarp) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (nt > 0 && warp == kVWarp) {
+    // ------------------------------------------------------------ V loads
     if (lane == 0) {
-      constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, false);
-      constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, true);
-      const uint32_t k_addr = smem_u32(smem + Ly::kK);
-      const uint32_t v_addr = smem_u32(smem + Ly::kV);
-      auto qk = [&](int t) {  // S_t = Q_t K^T
-        const uint32_t q_addr = smem_u32(smem + Ly::kQ + t * Ly::kQBytes);
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
-          mma_bf16(tmem_base + t * 128, smem_desc_sw128(q_addr + off, 16, 1024),
-                   smem_desc_sw128(k_addr + off, 16, 1024), idesc_qk, kk > 0);
+      prefetch_tensormap(&tm_vc);
+      prefetch_tensormap(&tm_vt);
+      // V_j -> slot j % kVStages, once both PV of V_{j - kVStages} completed
+      for (int j = 0; j < nt; ++j) {
+        const int st = j % kVStages;
+        if (j >= kVStages && !mbar_wait(&bars.v_empty[st], (j / kVStages - 1) & 1, abort)) {
+          fail();
+          break;
         }
-        mma_commit(&bars.s_full[t]);
-      };
-      auto pv = [&](int t, bool acc) {  // O_t (+)= P_t V
-        const uint32_t p_addr = smem_u32(smem + Ly::kP + t * Ly::kPBytes);
-#pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk) {
-          const uint32_t poff = (kk >> 2) * kPanelBytes + (kk & 3) * 32;
-          const uint32_t voff = kk * 16 * 128;  // 16 keys x 128-byte rows
-          mma_bf16(tmem_base + 256 + t * 128, smem_desc_sw128(p_addr + poff, 16, 1024),
-                   smem_desc_sw128(v_addr + voff, kPanelBytes, 1024), idesc_pv,
-                   (acc || kk > 0) ? 1u : 0u);
-        }
-        mma_commit(&bars.o_done[t]);
-      };
-      bool ok = mbar_wait(&bars.q_full, 0, abort) && mbar_wait(&bars.k_full, 0, abort);
-      if (ok) {
-        tc_fence_after();
-        qk(0);
-        if (has1) qk(1);
-        mma_commit(&bars.k_empty);
-      }
-      for (int j = 0; ok && j < nt; ++j) {
-        const bool next = j + 1 < nt;
-        ok = mbar_wait(&bars.v_full, j & 1, abort) && mbar_wait(&bars.p_full[0], j & 1, abort);
-        if (!ok) break;
-        tc_fence_after();
-        pv(0, j > 0);
-        if (next) {
-          ok = mbar_wait(&bars.k_full, (j + 1) & 1, abort) &&
-               mbar_wait(&bars.s_free[0], j & 1, abort);
-          if (!ok) break;
-          tc_fence_after();
-          qk(0);
-        }
-        if (has1) {
-          ok = mbar_wait(&bars.p_full[1], j & 1, abort);
-          if (!ok) break;
-          tc_fence_after();
-          pv(1, j > 0);
-        }
-        mma_commit(&bars.v_empty);
-        if (next) {
-          if (has1) {
-            ok = mbar_wait(&bars.s_free[1], j & 1, abort);
-            if (!ok) break;
-            tc_fence_after();
-            qk(1);
-          }
-          mma_commit(&bars.k_empty);
+        uint8_t* dst = smem + Ly::kV + st * Ly::kTileBytes;
+        mbar_arrive_expect_tx(&bars.v_full[st], Ly::kTileBytes);
+        for (int p = 0; p < Ly::kPanels; ++p) {
+          if (j < n_prefix)
+            tma_load_3d(dst + p * Ly::kKVPanel, &tm_vc, p * 64, (t_begin + j) * kBN,
+                        b * a.Hkv + g, &bars.v_full[st]);
+          else
+            tma_load_3d(dst + p * Ly::kKVPanel, &tm_vt, p * 64, g,
+                        b * a.N + (j - n_prefix) * kBN, &bars.v_full[st]);
         }
       }
-      if (!ok) fail();
     }
-  } else if (warp < kSoftWarps * ntiles) {
+  } else if (nt > 0 && warp == kMmaWarp) {
+    // ------------------------------------------------------------ MMA issuer
+    // QK^T runs one KV tile ahead of PV: for j: QK_{j+1}(t0), QK_{j+1}(t1) (each once
+    // that tile's softmax has read S_j), PV_j(t0), PV_j(t1) (P_j from TMEM).
+    // The whole warp runs this loop (wait outcomes made warp-uniform); one elected
+    // lane issues each MMA and commit.
+    constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, false);
+    constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, true);
+    const uint64_t q_desc0 = smem_desc_sw128(smem_u32(smem + Ly::kQ), 16, 1024);
+    const uint64_t k_desc0 = smem_desc_sw128(smem_u32(smem + Ly::kK), 16, 1024);
+    const uint64_t v_desc0 = smem_desc_sw128(smem_u32(smem + Ly::kV), Ly::kKVPanel, 1024);
+    auto wait = [&](uint64_t* bar, uint32_t parity) {
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(bar, parity, abort));
+      if (ok) tc_fence_after();
+      return ok;
+    };
+    // S_t = Q_t K_j^T
+    auto qk = [&](int t, int j) {
+      if (j >= 1 && !wait(&bars.s_free[t], (j - 1) & 1)) return false;
+      // descriptor start addresses are in 16-byte units in the low bits
+      const uint64_t qd = q_desc0 + ((t * Ly::kQBytes) >> 4);
+      const uint64_t kd = k_desc0 + (((j % kKStages) * Ly::kTileBytes) >> 4);
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t qo = ((kk >> 2) * Ly::kQPanel + (kk & 3) * 32) >> 4;
+        const uint32_t ko = ((kk >> 2) * Ly::kKVPanel + (kk & 3) * 32) >> 4;
+        mma_bf16_warp(tmem_base + t * 64, qd + qo, kd + ko, idesc_qk, kk > 0);
+      }
+      mma_commit_warp(&bars.s_full[t]);
+      return true;
+    };
+    // O_t (+)= P_t V_j, P_t read from TMEM (8 columns = 16 keys per step)
+    auto pv = [&](int t, int j) {
+      if (!wait(&bars.p_full[t], j & 1)) return false;
+      const uint64_t vd = v_desc0 + (((j % kVStages) * Ly::kTileBytes) >> 4);
+#pragma unroll
+      for (int kk = 0; kk < kBN / 16; ++kk)
+        mma_bf16_ts_warp(tmem_base + kTmemO + t * 128, tmem_base + kTmemP + t * 32 + kk * 8,
+                         vd + ((kk * 16 * kRowBytes) >> 4), idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+      mma_commit_warp(&bars.o_done[t]);
+      return true;
+    };
+    bool ok = wait(&bars.q_full, 0) && wait(&bars.k_full[0], 0) && qk(0, 0) && (!has1 || qk(1, 0));
+    if (ok) mma_commit_warp(&bars.k_empty[0]);
+    for (int j = 0; ok && j < nt; ++j) {
+      if (j + 1 < nt) {
+        ok = wait(&bars.k_full[(j + 1) % kKStages], ((j + 1) / kKStages) & 1) && qk(0, j + 1) &&
+             (!has1 || qk(1, j + 1));
+        if (!ok) break;
+        mma_commit_warp(&bars.k_empty[(j + 1) % kKStages]);
+      }
+      ok = wait(&bars.v_full[j % kVStages], (j / kVStages) & 1) && pv(0, j) && (!has1 || pv(1, j));
+      if (ok) mma_commit_warp(&bars.v_empty[j % kVStages]);
+    }
+    if (!ok && lane == 0) fail();
+  } else if (nt > 0 && warp < 4 * ntiles) {
     // ------------------------------------------------------------ softmax warps
-    const int t = warp / kSoftWarps;           // row tile
-    const int h = (warp % kSoftWarps) / 4;     // which 64 key columns / D/2 columns
-    const int quad = warp & 3;                 // TMEM lane quadrant
-    const int r = quad * 32 + lane;
+    const int t = warp >> 2;          // row tile
+    const int quad = warp & 3;        // TMEM lane quadrant
+    const int r = quad * 32 + lane;   // row of the tile
     const uint32_t lane_addr = static_cast<uint32_t>(quad * 32) << 16;
-    const uint32_t tS = tmem_base + t * 128 + h * 64 + lane_addr;
-    const uint32_t tO = tmem_base + 256 + t * 128 + h * (D / 2) + lane_addr;
-    uint8_t* sP = smem + Ly::kP + t * Ly::kPBytes + h * kPanelBytes;
+    const uint32_t tO = tmem_base + kTmemO + t * 128 + lane_addr;
+    const uint32_t tP = tmem_base + kTmemP + t * 32 + lane_addr;
     const int node = (mt0 + t) * nodes_per_tile + r / a.G;
     const int hh = r % a.G;
     const uint32_t* mrow =
@@ -401,86 +339,79 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
       // wait outcomes are made warp-uniform: tcgen05.ld needs the whole warp
-      const bool got = __all_sync(0xffffffffu, ok && mbar_wait(&bars.s_full[t], j & 1, abort));
-      uint32_t bits[2] = {0u, 0u};
-      float mx = -INFINITY;
-      if (got) {
-        tc_fence_after();
-        // masks: prefix keys beyond kv_len; tree keys outside the ancestor set
-        if (j < n_prefix) {
-          const int lim = kv - (t_begin + j) * kBN - h * 64;
-          bits[0] = lim >= 32 ? 0xffffffffu : (lim <= 0 ? 0u : (1u << lim) - 1u);
-          bits[1] = lim >= 64 ? 0xffffffffu : (lim <= 32 ? 0u : (1u << (lim - 32)) - 1u);
-        } else {
-          const int wi = (((j - n_prefix) * kBN) >> 5) + 2 * h;
-          bits[0] = (mrow && wi < a.W) ? __ldg(mrow + wi) : 0u;
-          bits[1] = (mrow && wi + 1 < a.W) ? __ldg(mrow + wi + 1) : 0u;
-        }
-        // pass 1: row max over this half's 64 columns, 32 at a time
-#pragma unroll 1
-        for (int c = 0; c < 2; ++c) {
-          float v[32];
-          tmem_ld32(tS + c * 32, v);
-          const uint32_t bc = c ? bits[1] : bits[0];
-          tmem_wait_ld();
-#pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if ((bc >> e) & 1u) mx = fmaxf(mx, v[e] * a.scale_log2);
-        }
-      }
-      // the two halves of each row meet here; a failed wait anywhere ends the loop
-      // for both (barrier with an AND reduction)
-      xchg[j & 1][t][h][r] = mx;
-      if (!bar_and(1 + t, kSoftThreads, got)) {
+      if (!__all_sync(0xffffffffu, mbar_wait(&bars.s_full[t], j & 1, abort))) {
         ok = false;
         break;
       }
-      mx = fmaxf(mx, xchg[j & 1][t][1 - h][r]);
+      tc_fence_after();
+      float v[64];
+      const uint32_t tS = tmem_base + t * 64 + lane_addr;
+      tmem_ld32(tS, *reinterpret_cast<float(*)[32]>(v));
+      tmem_ld32(tS + 32, *reinterpret_cast<float(*)[32]>(v + 32));
+      // masks: prefix keys beyond kv_len; tree keys outside the ancestor set (a
+      // full prefix tile needs none)
+      uint32_t b0, b1;
+      if (j < n_prefix) {
+        const int lim = kv - (t_begin + j) * kBN;
+        b0 = lim >= 32 ? 0xffffffffu : (lim <= 0 ? 0u : (1u << lim) - 1u);
+        b1 = lim >= 64 ? 0xffffffffu : (lim <= 32 ? 0u : (1u << (lim - 32)) - 1u);
+      } else {
+        const int wi = ((j - n_prefix) * kBN) >> 5;
+        b0 = (mrow && wi < a.W) ? __ldg(mrow + wi) : 0u;
+        b1 = (mrow && wi + 1 < a.W) ? __ldg(mrow + wi + 1) : 0u;
+      }
+      const bool full = j < n_prefix && kv - (t_begin + j) * kBN >= kBN;  // warp-uniform
+      tmem_wait_ld();
+      tc_fence_before();
+      mbar_arrive(&bars.s_free[t]);  // S_t may be overwritten by QK_{j+1}
+      if (!full) {  // masked scores -> -inf (exp2 of -inf is 0)
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          v[e] = ((b0 >> e) & 1u) ? v[e] : -INFINITY;
+          v[32 + e] = ((b1 >> e) & 1u) ? v[32 + e] : -INFINITY;
+        }
+      }
+      const float mx = row_max64(v) * a.scale_log2;  // scale > 0 commutes with max
       // stale-max online softmax: move m only when the row max exceeds it by > 2^8
       const bool move = mx > m + kRescaleLog2;
       const float alpha = move ? ex2(m - mx) : 1.f;
       if (move) m = mx;
       const float m_use = m == -INFINITY ? 0.f : m;
-      if (j > 0) {  // P buffer and O are free once PV_{j-1} of this tile completed
+      // p = exp2(s * scale - m); the row sum in four independent packed chains
+      const uint64_t sc2 = pack2(a.scale_log2, a.scale_log2), nm2 = pack2(-m_use, -m_use);
+      uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        float x0, x1;
+        unpack2(fma2(pack2(v[2 * i], v[2 * i + 1]), sc2, nm2), x0, x1);
+        v[2 * i] = ex2(x0);
+        v[2 * i + 1] = ex2(x1);
+        acc[i & 3] = add2(acc[i & 3], pack2(v[2 * i], v[2 * i + 1]));
+      }
+      float rs, rs1;
+      unpack2(add2(add2(acc[0], acc[1]), add2(acc[2], acc[3])), rs, rs1);
+      rs += rs1;
+      l = l * alpha + rs;
+      if (j > 0) {  // P_t and O_t are free once PV_{j-1} of this tile completed
         if (!__all_sync(0xffffffffu, mbar_wait(&bars.o_done[t], (j - 1) & 1, abort))) {
-          ok = false;  // leaves the loop at the next meeting point
-          continue;
+          ok = false;
+          break;
         }
         tc_fence_after();
       }
-      // pass 2: P = exp2(S*scale - m) for this half's 64 keys of row r, into its
-      // 64-key panel (bf16, 128-byte swizzle)
-      float rs = 0.f;
-#pragma unroll 1
-      for (int c = 0; c < 2; ++c) {
-        float v[32];
-        tmem_ld32(tS + c * 32, v);
-        const uint32_t bc = c ? bits[1] : bits[0];
-        tmem_wait_ld();
+      // row r of P_t (64 keys as 32 bf16 pairs) into this thread's TMEM lane
+      {
+        uint32_t pk[32];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          uint4 u;
-          uint32_t* w = reinterpret_cast<uint32_t*>(&u);
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int i0 = q * 8 + 2 * e;
-            const float p0 = ((bc >> i0) & 1u) ? ex2(fmaf(v[i0], a.scale_log2, -m_use)) : 0.f;
-            const float p1 =
-                ((bc >> (i0 + 1)) & 1u) ? ex2(fmaf(v[i0 + 1], a.scale_log2, -m_use)) : 0.f;
-            rs += p0 + p1;
-            const __nv_bfloat162 pv2 = __floats2bfloat162_rn(p0, p1);
-            w[e] = *reinterpret_cast<const uint32_t*>(&pv2);
-          }
-          const int chunk = c * 4 + q;
-          *reinterpret_cast<uint4*>(sP + r * 128 + ((chunk ^ (r & 7)) << 4)) = u;
+        for (int e = 0; e < 32; ++e) {
+          const __nv_bfloat162 pv2 = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+          pk[e] = *reinterpret_cast<const uint32_t*>(&pv2);
         }
+        tmem_st32(tP, *reinterpret_cast<const float(*)[32]>(pk));
       }
-      tc_fence_before();
-      mbar_arrive(&bars.s_free[t]);  // S_t may be overwritten by the next QK^T
-      l = l * alpha + rs;
       if (j > 0 && __any_sync(0xffffffffu, move)) {
-#pragma unroll
-        for (int c = 0; c < D / 64; ++c) {
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
           float o[32];
           tmem_ld32(tO + c * 32, o);
           tmem_wait_ld();
@@ -488,79 +419,154 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int e = 0; e < 32; ++e) o[e] *= alpha;
           tmem_st32(tO + c * 32, o);
         }
-        tmem_wait_st();
       }
-      fence_proxy_async();  // make the P stores visible to the tensor core
+      tmem_wait_st();  // P (and a rescaled O) are in TMEM before the MMA is released
       tc_fence_before();
       mbar_arrive(&bars.p_full[t]);
     }
-    // row sum = the two halves' sums (same running max)
-    lsum[t][h][r] = l;
-    const bool all_ok = bar_and(1 + t, kSoftThreads, ok);
-    l += lsum[t][1 - h][r];
-    ok = __all_sync(0xffffffffu, all_ok && mbar_wait(&bars.o_done[t], (nt - 1) & 1, abort));
-    if (ok) {
+    if (ok)
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars.o_done[t], (nt - 1) & 1, abort));
+    if (!ok) fail();
+    if (clustered) {
+      // this split's unnormalised row and (m, l) for the merge (a failed or empty
+      // row is marked by m = -inf and contributes nothing)
+      const size_t prow = static_cast<size_t>(blockIdx.x) * 2 * kBM + t * kBM + r;
+      a.part_ml[prow] = ok ? make_float2(m, l) : make_float2(-INFINITY, 0.f);
+      if (ok) {
+        tc_fence_after();
+        // column-quad-major, so a warp's 32 rows of one quad are 512 contiguous bytes
+        float4* dst = a.part_o + static_cast<size_t>(blockIdx.x) * (D / 4) * 2 * kBM + t * kBM + r;
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+          float o[32];
+          tmem_ld32(tO + c * 32, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            dst[(c * 8 + q) * 2 * kBM] = make_float4(o[q * 4], o[q * 4 + 1], o[q * 4 + 2], o[q * 4 + 3]);
+        }
+      }
+    } else if (ok) {
       tc_fence_after();
-      // epilogue, this half's D/2 columns, 32 at a time: the normalised bf16 row, or
-      // the fp32 partial left in this CTA's shared memory for the cluster merge.
-      // (clustered) the partial overwrites Q/K/V/P space: tile 0's rows cover Q and
-      // K, whose last readers (QK^T of both tiles) were issued before PV of tile 0
-      // and are therefore complete once its last o_done arrived; tile 1's rows are
-      // written after the last MMA of the CTA.  The other tile's P buffer lies
-      // beyond both.
+      // the normalised bf16 row, 32 columns at a time, and its lse
       const bool used = node < a.N && node < nn && l > 0.f;
       const float inv = used ? 1.f / l : 0.f;
       __nv_bfloat16* orow =
-          a.out + ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D + h * (D / 2);
-      float* prow = reinterpret_cast<float*>(smem) + (t * kBM + r) * kPartStride<D> + h * (D / 2);
+          a.out + ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
 #pragma unroll 1
-      for (int c = 0; c < D / 64; ++c) {
+      for (int c = 0; c < D / 32; ++c) {
         float o[32];
         tmem_ld32(tO + c * 32, o);
         tmem_wait_ld();
-        if (!clustered) {
-          if (node < a.N) {
+        if (node < a.N) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              uint4 u;
-              uint32_t* w = reinterpret_cast<uint32_t*>(&u);
+          for (int q = 0; q < 4; ++q) {
+            uint4 w4;
+            uint32_t* w = reinterpret_cast<uint32_t*>(&w4);
 #pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const __nv_bfloat162 o2 =
-                    __floats2bfloat162_rn(o[q * 8 + 2 * e] * inv, o[q * 8 + 2 * e + 1] * inv);
-                w[e] = *reinterpret_cast<const uint32_t*>(&o2);
-              }
-              *reinterpret_cast<uint4*>(orow + c * 32 + q * 8) = u;
+            for (int e = 0; e < 4; ++e) {
+              const __nv_bfloat162 o2 =
+                  __floats2bfloat162_rn(o[q * 8 + 2 * e] * inv, o[q * 8 + 2 * e + 1] * inv);
+              w[e] = *reinterpret_cast<const uint32_t*>(&o2);
             }
+            *reinterpret_cast<uint4*>(orow + c * 32 + q * 8) = w4;
           }
-        } else {
-#pragma unroll
-          for (int q = 0; q < 8; ++q)
-            *reinterpret_cast<float4*>(prow + c * 32 + q * 4) =
-                make_float4(o[q * 4], o[q * 4 + 1], o[q * 4 + 2], o[q * 4 + 3]);
         }
       }
-      if (h == 0) {
-        if (!clustered) {
-          if (node < a.N && a.lse)
-            a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] =
-                used ? (m + log2f(l)) * kLn2 : -INFINITY;
-        } else {
-          part_ml[t][r] = make_float2(m, l);
-        }
-      }
-    } else {
-      fail();
-      if (clustered && h == 0) part_ml[t][r] = make_float2(-INFINITY, 0.f);
+      if (node < a.N && a.lse)
+        a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] =
+            used ? (m + log2f(l)) * kLn2 : -INFINITY;
     }
   }
+
+  if (!clustered) {
+    if (nt == 0 && tid < ntiles * kBM) {  // no keys at all: a zero row, lse -inf
+      const int t = tid / kBM, r = tid % kBM;
+      const int node = (mt0 + t) * nodes_per_tile + r / a.G, hh = r % a.G;
+      if (node < a.N) {
+        __nv_bfloat16* orow =
+            a.out + ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
+        for (int c = 0; c < D; c += 8) *reinterpret_cast<uint4*>(orow + c) = make_uint4(0, 0, 0, 0);
+        if (a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = -INFINITY;
+      }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+      tc_fence_after();
+      tmem_dealloc(tmem_base, kTmemCols);
+    }
+    return;
+  }
+
+  // ---------------------------------------------------------------- split merge
+  // The KV splits of this row block are the CTAs of the cluster; each has left its
+  // rows' (m, l) and unnormalised O in the workspace.  Rows are dealt out in slices,
+  // one per CTA, and each CTA combines its slice over the splits with log-sum-exp
+  // weights (the partials stay in L2).
+  if (nt == 0 && tid < ntiles * kBM)  // an empty split contributes nothing
+    a.part_ml[static_cast<size_t>(blockIdx.x) * 2 * kBM + tid] = make_float2(-INFINITY, 0.f);
   tc_fence_before();
   __syncthreads();
   if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem_base, kTmemCols);
   }
-  if (clustered) cluster_merge<D>(a, b, g, mt0, ntiles, nn, smem, part_ml);
+  // release / acquire at cluster scope: every split's partial rows are visible
+  cg::this_cluster().sync();
+  const int R = ntiles * kBM;
+  const int nsp = a.n_splits;
+  const int slice = (R + nsp - 1) / nsp;
+  const size_t cta0 = static_cast<size_t>(blockIdx.x - split);  // first CTA of the cluster
+  const int r0 = split * slice;
+  const int nr = max(0, min(R, r0 + slice) - r0);
+  constexpr int kC4 = D / 4;  // float4 columns per row
+  // one item = one row of the slice x one column quad; all its loads (every split's
+  // (m, l) and partial) are issued together, so the merge costs one L2 round trip
+  for (int item = tid; item < nr * kC4; item += kThreads) {
+    const int c4 = item / nr, i = item % nr;  // rows fastest: coalesced partial loads
+    const int row = r0 + i;
+    const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
+    const int hh = (row % kBM) % a.G;
+    if (node >= a.N) continue;
+    float2 ml[kMaxSplits];
+    float4 o[kMaxSplits];
+#pragma unroll
+    for (int s = 0; s < kMaxSplits; ++s) {
+      const bool in = s < nsp;
+      ml[s] = in ? __ldcg(a.part_ml + (cta0 + s) * 2 * kBM + row) : make_float2(-INFINITY, 0.f);
+      o[s] = in ? __ldcg(a.part_o + ((cta0 + s) * kC4 + c4) * 2 * kBM + row)
+                : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    float M = -INFINITY;
+#pragma unroll
+    for (int s = 0; s < kMaxSplits; ++s) M = fmaxf(M, ml[s].x);
+    float L = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int s = 0; s < kMaxSplits; ++s) {
+      // a split without keys for the row (m = -inf) wrote no O: weight 0, value unused
+      if (M == -INFINITY || ml[s].x == -INFINITY) continue;
+      const float w = ex2(ml[s].x - M);
+      L += ml[s].y * w;
+      acc.x += w * o[s].x;
+      acc.y += w * o[s].y;
+      acc.z += w * o[s].z;
+      acc.w += w * o[s].w;
+    }
+    const bool used = node < nn && L > 0.f;
+    const float inv = used ? 1.f / L : 0.f;
+    const size_t orow = ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
+    const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+    uint2 u2;
+    u2.x = *reinterpret_cast<const uint32_t*>(&lo);
+    u2.y = *reinterpret_cast<const uint32_t*>(&hi);
+    *reinterpret_cast<uint2*>(a.out + orow + c4 * 4) = u2;
+    if (c4 == 0 && a.lse)
+      a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] =
+          used ? (M + log2f(L)) * kLn2 : -INFINITY;
+  }
 }
 
 // ------------------------------------------------------------------ host side
@@ -608,20 +614,21 @@ Plan make_plan(int B, int N, int Hq, int Hkv, int Tmax, const int* active) {
   int max_splits = prefix_tiles / 2 > 1 ? prefix_tiles / 2 : 1;
   if (max_splits > kMaxSplits) max_splits = kMaxSplits;
   // Choose row tiles per CTA (2 lets the softmax of one tile hide behind the
-  // tensor-core work of the other) and the split count by the estimated time:
-  // waves of resident clusters x (KV tiles per CTA x cost of one KV tile + fixed
-  // cost), lightly penalising splits (each adds rows to merge).
+  // tensor-core work of the other, and reads K/V once for both) and the split
+  // count by the estimated time: waves of resident clusters x (KV tiles per CTA x
+  // cost of one KV tile + fixed cost), lightly penalising splits (each adds rows
+  // to merge).
   double best_cost = 1e30;
   p.tpc = 1;
   p.n_splits = 1;
   for (int tpc = 1; tpc <= 2; ++tpc) {
     const int groups = (p.n_mt + tpc - 1) / tpc;
     const long long units = static_cast<long long>(B) * Hkv * groups;
-    const double tile_cost = tpc == 2 ? 1.15 : 1.0;
+    const double tile_cost = tpc == 2 ? 1.3 : 1.0;
     for (int s = 1; s <= max_splits; ++s) {
       if (active[s] < 1) continue;
       const double waves = std::ceil(static_cast<double>(units) / active[s]);
-      const double work = (prefix_tiles + 1.0) / s * tile_cost + 1.5;
+      const double work = (prefix_tiles + 2.0) / s * tile_cost + 3.0;
       const double cost = waves * work * (1.0 + 0.02 * (s - 1));
       if (cost < best_cost - 1e-9) {
         best_cost = cost;
@@ -689,10 +696,13 @@ const int* active_clusters() {
 using namespace presto;
 
 extern "C" size_t presto_attn_workspace(int B, int N, int Hq, int Hkv, int D, int Tmax) {
-  if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || Tmax < 0 || (D != 64 && D != 128))
+  if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || Tmax < 1 || (D != 64 && D != 128))
     return 0;
-  // KV splits merge inside thread-block clusters; no device workspace is needed.
-  return 256;
+  // KV splits leave fp32 partial rows and (m, l) for the in-kernel merge
+  const int* active = D == 128 ? active_clusters<128>() : active_clusters<64>();
+  const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
+  if (p.n_splits == 1) return 256;
+  return align_up(p.ctas * 2 * kBM * (static_cast<size_t>(D) * 4 + 8), 256);
 }
 
 extern "C" int presto_tree_attention(const void* q, const void* k_cache, const void* v_cache,
@@ -714,9 +724,13 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
     PRESTO_CHECK_ARG(reinterpret_cast<uintptr_t>(p) % 16 == 0);
   const int* active = D == 128 ? active_clusters<128>() : active_clusters<64>();
   const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
-  (void)ws;
-  (void)ws_bytes;
   Args a{};
+  if (p.n_splits > 1) {
+    const size_t need = p.ctas * 2 * kBM * (static_cast<size_t>(D) * 4 + 8);
+    if (!ws || reinterpret_cast<uintptr_t>(ws) % 16 || ws_bytes < need) return PRESTO_ERR_WORKSPACE;
+    a.part_o = static_cast<float4*>(ws);
+    a.part_ml = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.ctas * 2 * kBM * D * 4);
+  }
   const uint64_t e = 2;  // bf16 bytes
   CUtensorMap tq, tkc, tvc, tkt, tvt;
   const uint64_t Du = static_cast<uint64_t>(D);

@@ -53,47 +53,58 @@ class DraftVerifyStep:
 
     CALLS = ("topk", "build", "mask", "attention", "accept")
 
-    def run(self, logits, ctx2, layers, kv_len, target_token, stream=None, marks=None):
+    def run(self, logits, ctx2, layers, kv_len, target_token, stream=None, marks=None,
+            only=None):
         """One round.  `layers` is a list of dicts with q, k_cache, v_cache, k_tree,
         v_tree (one per attention layer).  Results stay in the step's buffers.
         `marks` (optional) maps a call name to a (start, end) pair of CUDA events
-        recorded around that call on the launch stream."""
+        recorded around that call on the launch stream.  `only` (optional) names
+        the calls to make; the others are skipped and their results are whatever
+        the buffers hold from an earlier round (for timing one call alone)."""
         s = torch.cuda.current_stream(self.device) if stream is None else stream
 
         def mark(name, i):
             if marks is not None and name in marks:
                 marks[name][i].record(s)
 
-        mark("topk", 0)
-        P.presto_topk(logits, self.k, self.topk_ids, self.topk_logq, self.lse, ws=self.ws_topk,
-                      dev_status=self.dev_status, stream=s)
-        mark("topk", 1)
-        mark("build", 0)
-        P.presto_score_build_tree(self.topk_ids, self.topk_logq, ctx2, self.ngram, self.lam,
-                                  self.N, b=self.b, out=self.tree, ws=self.ws_build,
-                                  dev_status=self.dev_status, stream=s)
-        mark("build", 1)
-        mark("mask", 0)
-        P.presto_tree_mask(self.tree["parent"], self.tree["depth"], self.tree["n_nodes"], kv_len,
-                           self.mask, self.pos_ids, dev_status=self.dev_status, stream=s)
-        mark("mask", 1)
-        mark("attention", 0)
-        for lay in layers:
-            P.presto_tree_attention(lay["q"], lay["k_cache"], lay["v_cache"], kv_len,
-                                    lay["k_tree"], lay["v_tree"], self.mask,
-                                    self.tree["n_nodes"], out=self.attn_out, lse=self.attn_lse,
-                                    ws=self.ws_attn, dev_status=self.dev_status, stream=s)
-        mark("attention", 1)
-        mark("accept", 0)
-        P.presto_accept(self.tree["token"], self.tree["parent"], self.tree["depth"], self.mask,
-                        self.tree["n_nodes"], target_token, self.L, self.accept_len,
-                        self.accept_path, self.bonus, dev_status=self.dev_status, stream=s)
-        mark("accept", 1)
+        def on(name):
+            return only is None or name in only
+
+        if on("topk"):
+            mark("topk", 0)
+            P.presto_topk(logits, self.k, self.topk_ids, self.topk_logq, self.lse, ws=self.ws_topk,
+                          dev_status=self.dev_status, stream=s)
+            mark("topk", 1)
+        if on("build"):
+            mark("build", 0)
+            P.presto_score_build_tree(self.topk_ids, self.topk_logq, ctx2, self.ngram, self.lam,
+                                      self.N, b=self.b, out=self.tree, ws=self.ws_build,
+                                      dev_status=self.dev_status, stream=s)
+            mark("build", 1)
+        if on("mask"):
+            mark("mask", 0)
+            P.presto_tree_mask(self.tree["parent"], self.tree["depth"], self.tree["n_nodes"], kv_len,
+                               self.mask, self.pos_ids, dev_status=self.dev_status, stream=s)
+            mark("mask", 1)
+        if on("attention"):
+            mark("attention", 0)
+            for lay in layers:
+                P.presto_tree_attention(lay["q"], lay["k_cache"], lay["v_cache"], kv_len,
+                                        lay["k_tree"], lay["v_tree"], self.mask,
+                                        self.tree["n_nodes"], out=self.attn_out, lse=self.attn_lse,
+                                        ws=self.ws_attn, dev_status=self.dev_status, stream=s)
+            mark("attention", 1)
+        if on("accept"):
+            mark("accept", 0)
+            P.presto_accept(self.tree["token"], self.tree["parent"], self.tree["depth"], self.mask,
+                            self.tree["n_nodes"], target_token, self.L, self.accept_len,
+                            self.accept_path, self.bonus, dev_status=self.dev_status, stream=s)
+            mark("accept", 1)
 
     def kernels_per_round(self, n_layers=1):
-        """Library kernels one round launches (the split-KV combine adds one per layer)."""
-        splits = self.ws_attn.numel() > 256
-        return 4 + n_layers * (2 if splits else 1)
+        """Library kernels one round launches: top-k, tree build, mask, accept and
+        one attention kernel per layer (KV splits merge inside the kernel)."""
+        return 4 + n_layers
 
     def capture(self, logits, ctx2, layers, kv_len, target_token):
         """Capture one round on these exact input tensors into a CUDA graph."""

@@ -88,9 +88,12 @@ int presto_version(void);
  *               descending order; equal values are ordered by lower token id.
  *   topk_logq   [B, L, k] float32 out: log q_d(t) = x_t - log sum_v exp(x_v).
  *   lse         [B, L] float32 out, nullable: log sum_v exp(x_v).
- *   ws          presto_topk_workspace(B, L, V, k) bytes.
+ *   ws          presto_topk_workspace(B, L, V, k) bytes (currently 256 for every
+ *               shape and unused: a row's spans merge inside one thread-block
+ *               cluster; the argument is kept so that a plan may use it).
  *   dev_status  nullable; PRESTO_DEV_NONFINITE when a row has no finite maximum.
- * One pass over the logits; accumulation in float32.
+ * One pass over the logits; accumulation in float32.  The base pointer must be
+ * aligned to the element size; rows need not be 16-byte aligned.
  */
 size_t presto_topk_workspace(int B, int L, int V, int k);
 int presto_topk(const void* logits, int dtype, int B, int L, int V, long long row_stride,
@@ -101,11 +104,12 @@ int presto_topk(const void* logits, int dtype, int B, int L, int V, long long ro
  * presto_topk_noalloc - presto_topk for callers that cannot allocate device memory.
  * The paper has no counterpart; this is a deployment variant of presto_topk.
  *
- * Same arguments and results as presto_topk, without the workspace: the span
- * partials live in a file-scope device array of PRESTO_TOPK_STATIC_SCRATCH_BYTES
- * (16 KiB) that every GPU loading this library keeps for the life of the process.
- * Returns PRESTO_ERR_UNSUPPORTED, enqueueing nothing, when
- * presto_topk_workspace(B, L, V, k) exceeds that size.  Calls no cudaMalloc or
+ * Same arguments and results as presto_topk, without the workspace: whatever
+ * scratch the plan needs lives in a file-scope device array of
+ * PRESTO_TOPK_STATIC_SCRATCH_BYTES (16 KiB) that every GPU loading this library
+ * keeps for the life of the process.  Returns PRESTO_ERR_UNSUPPORTED, enqueueing
+ * nothing, when presto_topk_workspace(B, L, V, k) exceeds that size (no shape does
+ * with the current plan).  Calls no cudaMalloc or
  * cudaFree.  The first call on a device looks up the array's device address
  * (cudaGetSymbolAddress, with that device current) and caches it; make that
  * first call before any stream capture.  All calls on a device share the one

@@ -164,9 +164,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ntiles = has1 ? 2 : 1;
   const bool clustered = a.n_splits > 1;
   const int nodes_per_tile = kBM / a.G;
-  // the sequence's lengths: loaded now, used after the set-up below
-  const int kv_raw = a.kv_len[b];
-  const int nn_raw = a.n_nodes[b];
+  pdl_launch_dependents();
 
   if (tid == 0) {
     mbar_init(&bars.q_full, 1);
@@ -194,6 +192,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait();  // the mask and node counts come from the previous kernels on the stream
+  const int kv_raw = a.kv_len[b];
+  const int nn_raw = a.n_nodes[b];
 
   int kv = kv_raw;
   if (kv < 0 || kv > a.Tmax) {
@@ -767,13 +768,14 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
   cfg.gridDim = dim3(static_cast<unsigned>(p.ctas));
   cfg.blockDim = dim3(kThreads);
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = p.n_splits;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1] = pdl_attribute();
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   cudaError_t err;
   if (D == 128) {
     set_smem_attr<128>();

@@ -336,6 +336,7 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
 
 __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   namespace cg = cooperative_groups;
+  pdl_launch_dependents();
   extern __shared__ __align__(16) unsigned char dyn[];
   __shared__ Smem sm;
   cg::cluster_group cluster = cg::this_cluster();
@@ -355,7 +356,8 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   const size_t stage_off = a.tables_in_smem ? tl.bytes : 0;
   float* st_s = reinterpret_cast<float*>(dyn + stage_off);
 
-  // ---- candidates and context
+  // ---- candidates and context (produced by the previous kernel on the stream)
+  pdl_wait();
   for (int i = tid; i < L * k; i += kThreads) {
     const int d = i / k, j = i - d * k;
     int t = a.ids[(static_cast<size_t>(b) * L + d) * k + j];
@@ -595,13 +597,14 @@ extern "C" int presto_score_build_tree(const int32_t* topk_ids, const float* top
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = kCluster;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1] = pdl_attribute();
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   if (cudaLaunchKernelEx(&cfg, build_kernel, a) != cudaSuccess) return PRESTO_ERR_CUDA;
   return launch_status();
 }

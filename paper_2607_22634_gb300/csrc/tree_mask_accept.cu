@@ -20,6 +20,8 @@ __global__ void __launch_bounds__(kMaxN) mask_kernel(const int32_t* node_parent,
   __shared__ int par[kMaxN];
   __shared__ int dep[kMaxN];
   __shared__ uint32_t rows[kMaxN][kMaxW + 1];
+  pdl_launch_dependents();
+  pdl_wait();  // the tree comes from the previous kernel on the stream
   const int b = blockIdx.x, i = threadIdx.x;
   int n = n_nodes[b];
   if (n < 1 || n > N) {
@@ -67,6 +69,8 @@ __global__ void __launch_bounds__(32) accept_kernel(
     const int32_t* node_token, const int32_t* node_parent, const int32_t* node_depth,
     const uint32_t* mask, const int32_t* n_nodes, const int32_t* target_token, int N, int W,
     int L, int32_t* accept_len, int32_t* accept_path, int32_t* bonus, int32_t* dev_status) {
+  pdl_launch_dependents();
+  pdl_wait();  // the tree and the target tokens come from earlier kernels on the stream
   const int b = blockIdx.x, lane = threadIdx.x;
   int n = n_nodes[b];
   if (n < 1 || n > N) {
@@ -146,8 +150,16 @@ extern "C" int presto_tree_mask(const int32_t* node_parent, const int32_t* node_
   PRESTO_CHECK_LIMIT(N <= kMaxN);
   const int W = (N + 31) / 32;
   const int threads = (N + 31) / 32 * 32;
-  mask_kernel<<<B, threads, 0, stream>>>(node_parent, node_depth, n_nodes, kv_len, N, W, mask,
-                                         pos_ids, dev_status);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(B));
+  cfg.blockDim = dim3(static_cast<unsigned>(threads));
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1] = {pdl_attribute()};
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, mask_kernel, node_parent, node_depth, n_nodes, kv_len, N, W, mask,
+                         pos_ids, dev_status) != cudaSuccess)
+    return PRESTO_ERR_CUDA;
   return launch_status();
 }
 
@@ -161,8 +173,16 @@ extern "C" int presto_accept(const int32_t* node_token, const int32_t* node_pare
   PRESTO_CHECK_ARG(B >= 1 && N >= 1 && L >= 1);
   PRESTO_CHECK_LIMIT(N <= kMaxN && L <= kMaxL);
   const int W = (N + 31) / 32;
-  accept_kernel<<<B, 32, 0, stream>>>(node_token, node_parent, node_depth, mask, n_nodes,
-                                      target_token, N, W, L, accept_len, accept_path, bonus,
-                                      dev_status);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(B));
+  cfg.blockDim = dim3(32);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1] = {pdl_attribute()};
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (cudaLaunchKernelEx(&cfg, accept_kernel, node_token, node_parent, node_depth, mask, n_nodes,
+                         target_token, N, W, L, accept_len, accept_path, bonus,
+                         dev_status) != cudaSuccess)
+    return PRESTO_ERR_CUDA;
   return launch_status();
 }

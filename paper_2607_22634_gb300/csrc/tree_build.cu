@@ -107,7 +107,8 @@ struct Smem {
   int cid[kMaxL][kMaxK];          // candidate tokens of every depth
   float clq[kMaxL][kMaxK];        // their log q
   int ctx0, ctx1;
-  int nc;                         // candidates of the current level (phase 2)
+  int nc[2];                      // candidates of a level (phase 2, double-buffered)
+  unsigned long long tau;         // the smallest key of a full A (phase 2)
 };
 
 // Tables of one sequence, indexed by context c = d * ctx_stride + ci (d = depth of
@@ -155,8 +156,8 @@ constexpr size_t kDynSmemBudget = 200 * 1024;
 constexpr int kCluster = 8;
 
 // Phase-2 scratch of the leader CTA (aliases the phase-1 staging area).  The kept
-// set A (non-root nodes, sorted by key, so A[r] is node r + 1) is double-buffered;
-// C holds one level's candidates.  Per entry: key, the index of its own children's
+// set A (non-root nodes, sorted by key, so A[r] is node r + 1) and the candidate
+// set C of a level are double-buffered.  Per entry: key, the index of its own children's
 // context (kNoCtx at depth L), its candidate index j, and its parent's node index.
 struct P2Layout {
   size_t akey, axc, apid, aj, ckey, cxc, cpid, cj, rk, bytes;
@@ -164,14 +165,14 @@ struct P2Layout {
     const size_t na = N, nc = static_cast<size_t>(N) * bf;
     size_t o = 0;
     akey = o;  o += 2 * na * 8;
-    ckey = o;  o += nc * 8;
+    ckey = o;  o += 2 * nc * 8;
     axc = o;   o += 2 * na * 4;
-    cxc = o;   o += nc * 4;
+    cxc = o;   o += 2 * nc * 4;
     apid = o;  o += align_up(2 * na * 2, 4);
-    cpid = o;  o += align_up(nc * 2, 4);
+    cpid = o;  o += align_up(2 * nc * 2, 4);
     rk = o;    o += align_up((na + nc) * 2, 4);
     aj = o;    o += align_up(2 * na, 4);
-    cj = o;    o += align_up(nc, 4);
+    cj = o;    o += align_up(2 * nc, 4);
     bytes = align_up(o, 16);
   }
 };
@@ -195,75 +196,60 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
   const int L = a.L, k = a.k, N = a.N, nb = a.bf;
   const int cs = a.use_table ? k * k : 1;
   const int cap = N - 1;  // non-root nodes
+  const int lane = tid & 31;
   const P2Layout ly(N, nb);
-  // A buffer b of each field starts at b * N
+  const int NC = N * nb;
+  // buffer u of each A field starts at u * N, of each C field at u * N * nb
   uint64_t* const akey = reinterpret_cast<uint64_t*>(p2 + ly.akey);
   uint32_t* const axc = reinterpret_cast<uint32_t*>(p2 + ly.axc);
   int16_t* const apid = reinterpret_cast<int16_t*>(p2 + ly.apid);
   uint8_t* const aj = p2 + ly.aj;
-  uint64_t* ckey = reinterpret_cast<uint64_t*>(p2 + ly.ckey);
-  uint32_t* cxc = reinterpret_cast<uint32_t*>(p2 + ly.cxc);
-  int16_t* cpid = reinterpret_cast<int16_t*>(p2 + ly.cpid);
-  uint8_t* cj = p2 + ly.cj;
-  int16_t* rk = reinterpret_cast<int16_t*>(p2 + ly.rk);
+  uint64_t* const ckey = reinterpret_cast<uint64_t*>(p2 + ly.ckey);
+  uint32_t* const cxc = reinterpret_cast<uint32_t*>(p2 + ly.cxc);
+  int16_t* const cpid = reinterpret_cast<int16_t*>(p2 + ly.cpid);
+  uint8_t* const cj = p2 + ly.cj;
+  int16_t* const rk = reinterpret_cast<int16_t*>(p2 + ly.rk);
 
-  if (tid == 0) sm.nc = 0;
-  __syncthreads();
-  int na = 0, cur = 0;
-  uint64_t tau = 0ull;  // candidates need key > tau (0: A not yet full)
-  for (int d = 0; d < L && cap > 0; ++d) {
-    // ---- candidates of depth d + 1: children of the root (d = 0) or of A's
-    // depth-d nodes
-    const int parents = d == 0 ? 1 : na;
-    for (int q = tid; q < parents * nb; q += kThreads) {
-      const int e = q / nb, c = q - e * nb;
-      uint32_t x;
-      float Sp;
-      int pnode, pj;
-      if (d == 0) {
-        x = 0u;
-        Sp = 0.f;
-        pnode = 0;
-        pj = 0;
-      } else {
-        const uint64_t ke = akey[cur * N + e];
-        if (63 - static_cast<int>((ke >> 26) & 63u) != d) continue;
-        x = axc[cur * N + e];
-        if (x == kNoCtx) continue;
-        Sp = unordered(static_cast<uint32_t>(ke >> 32));
-        pnode = e + 1;
-        pj = aj[cur * N + e];
-      }
-      const uint2 kd = kids[x * nb + c];
-      const uint64_t key =
-          (static_cast<uint64_t>(ordered(__fadd_rn(Sp, __uint_as_float(kd.x)))) << 32) |
+  // Child c of a node with score Sp, children context x, candidate index pj and
+  // node index pnode, at depth dc: its key, context and candidate index.
+  auto child = [&](uint32_t x, float Sp, int pj, int pnode, int dc, int c, uint64_t& key,
+                   uint32_t& xc, int& jc) {
+    const uint2 kd = kids[x * nb + c];
+    key = (static_cast<uint64_t>(ordered(__fadd_rn(Sp, __uint_as_float(kd.x)))) << 32) |
           (kd.y & ~0xFFu) | static_cast<uint32_t>(255 - pnode);
-      if (key <= tau) continue;
-      const int jc = static_cast<int>(kd.y & 0xFFu);
-      const int dc = d + 1;
-      const uint32_t xc = dc >= L ? kNoCtx
-                                  : static_cast<uint32_t>(
-                                        dc * cs + (!a.use_table ? 0 : (dc == 1 ? jc : pj * k + jc)));
-      const int slot = atomicAdd(&sm.nc, 1);
-      ckey[slot] = key;
-      cxc[slot] = xc;
-      cpid[slot] = static_cast<int16_t>(pnode);
-      cj[slot] = static_cast<uint8_t>(jc);
-    }
-    __syncthreads();
-    const int m = sm.nc;
-    if (m == 0) break;  // no node of depth d + 1 can be kept: none deeper either
+    jc = static_cast<int>(kd.y & 0xFFu);
+    xc = dc >= L ? kNoCtx
+                 : static_cast<uint32_t>(dc * cs + (!a.use_table ? 0 : (dc == 1 ? jc : pj * k + jc)));
+  };
+
+  // level 1: the root's children (A is empty, so every one is a candidate)
+  if (cap > 0 && tid < nb) {
+    uint64_t key;
+    uint32_t xc;
+    int jc;
+    child(0u, 0.f, 0, 0, 1, tid, key, xc, jc);
+    ckey[tid] = key;
+    cxc[tid] = xc;
+    cpid[tid] = 0;
+    cj[tid] = static_cast<uint8_t>(jc);
+  }
+  if (tid == 0) sm.nc[1] = 0;
+  __syncthreads();
+  int na = 0, m = cap > 0 ? nb : 0, cur = 0, cc = 0;
+  uint64_t tau = 0ull;  // candidates need key > tau (0: A not yet full)
+  for (int step = 0; m > 0; ++step) {
     // ---- ranks in A u C by (key desc, position asc); A is sorted
+    const uint64_t* C = ckey + cc * NC;
     const int ne = na + m;
     for (int e = tid; e < ne; e += kThreads) {
       int r;
       if (e < na) {
         const uint64_t ke = akey[cur * N + e];
         r = e;
-        for (int i = 0; i < m; ++i) r += ckey[i] > ke;
+        for (int i = 0; i < m; ++i) r += C[i] > ke;
       } else {
         const int ci = e - na;
-        const uint64_t ke = ckey[ci];
+        const uint64_t ke = C[ci];
         int lo = 0, hi = na;  // A entries with key >= ke
         while (lo < hi) {
           const int mid = (lo + hi) >> 1;
@@ -272,15 +258,20 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
         }
         r = lo;
         for (int i = 0; i < m; ++i) {
-          const uint64_t ki = ckey[i];
+          const uint64_t ki = C[i];
           r += ki > ke || (ki == ke && i < ci);
         }
       }
       rk[e] = static_cast<int16_t>(r < cap ? r : cap);
+      if (r == cap - 1) sm.tau = e < na ? akey[cur * N + e] : C[e - na];  // the new A's last key
     }
+    if (tid == 0) sm.nc[cc ^ 1] = 0;  // the next level's counter (last read a level ago)
     __syncthreads();
-    // ---- the cap largest become the new A; parent indices follow their ranks
-    const int nxt = cur ^ 1;
+    if (ne >= cap) tau = sm.tau;  // the new A is full: its smallest key
+    // ---- the cap largest become the new A (parent indices follow their ranks), and
+    // the new nodes, the survivors of C, generate the next level's candidates: their
+    // children with key > tau, the smallest key of the new A once it is full
+    const int nxt = cur ^ 1, cn = cc ^ 1;
     for (int e = tid; e < ne; e += kThreads) {
       const int r = rk[e];
       if (r >= cap) continue;
@@ -291,10 +282,10 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
         aj[nxt * N + r] = aj[cur * N + e];
         pid = apid[cur * N + e];
       } else {
-        akey[nxt * N + r] = ckey[e - na];
-        axc[nxt * N + r] = cxc[e - na];
-        aj[nxt * N + r] = cj[e - na];
-        pid = cpid[e - na];
+        akey[nxt * N + r] = C[e - na];
+        axc[nxt * N + r] = cxc[cc * NC + e - na];
+        aj[nxt * N + r] = cj[cc * NC + e - na];
+        pid = cpid[cc * NC + e - na];
       }
       if (pid > 0) {
         const int pr = rk[pid - 1];
@@ -303,11 +294,40 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
       }
       apid[nxt * N + r] = static_cast<int16_t>(pid);
     }
-    if (tid == 0) sm.nc = 0;  // every thread read it before the last barrier
+    // (candidate, child) pairs over the whole CTA; slots reserved per warp
+    const int pairs = m * nb;
+    const int iters = (pairs + kThreads - 1) / kThreads;  // uniform, for the warp scans
+    for (int it = 0; it < iters; ++it) {
+      const int q = it * kThreads + tid;
+      const int ci = q / nb, c = q - ci * nb;
+      const int r = q < pairs ? rk[na + ci] : cap;
+      const uint32_t xe = r < cap ? cxc[cc * NC + ci] : kNoCtx;
+      uint64_t key = 0ull;
+      uint32_t xc = kNoCtx;
+      int jc = 0;
+      if (xe != kNoCtx) {  // a new node below depth L
+        const uint64_t ke = C[ci];
+        const int dc = 64 - static_cast<int>((ke >> 26) & 63u);  // the children's depth
+        child(xe, unordered(static_cast<uint32_t>(ke >> 32)), cj[cc * NC + ci], r + 1, dc, c,
+              key, xc, jc);
+      }
+      const bool keep = key > tau;
+      const unsigned bal = __ballot_sync(0xffffffffu, keep);
+      int base = 0;
+      if (lane == 0 && bal) base = atomicAdd(&sm.nc[cn], __popc(bal));
+      base = __shfl_sync(0xffffffffu, base, 0) + __popc(bal & ((1u << lane) - 1u));
+      if (keep) {
+        ckey[cn * NC + base] = key;
+        cxc[cn * NC + base] = xc;
+        cpid[cn * NC + base] = static_cast<int16_t>(r + 1);
+        cj[cn * NC + base] = static_cast<uint8_t>(jc);
+      }
+    }
     na = ne < cap ? ne : cap;
     cur = nxt;
+    cc = cn;
     __syncthreads();
-    if (na == cap) tau = akey[cur * N + cap - 1];
+    m = sm.nc[cc];
   }
   // ---- write the tree: node 0 is the root, node r + 1 is A[r]
   for (int i = tid; i < N; i += kThreads) {
@@ -385,7 +405,11 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   const int g0 = rank * a.per_cta;
   const int g1 = min(a.nctx_all, g0 + a.per_cta);
   const int my = g1 > g0 ? (g1 - g0) * k : 0;
-  constexpr int kBatch = 4;
+  // each probe first reads its home slot (key and value); the probes that meet
+  // another key (about a quarter at the tables' load factor) then read the next kWin
+  // slots in one round; only a longer chain continues slot by slot
+  constexpr int kBatch = 2;
+  constexpr int kWin = 4;
   for (int f0 = tid; f0 < my; f0 += kThreads * kBatch) {
     uint64_t key[kBatch];
     uint32_t h[kBatch];
@@ -418,13 +442,26 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
                static_cast<uint64_t>(sm.cid[d][j] & 0x3FFFF);
       h[q] = static_cast<uint32_t>(fmix64(key[q])) & a.cap_mask;
     }
-    uint64_t kv[kBatch];
-    float vv[kBatch];
+    uint64_t k0[kBatch];
+    float v0[kBatch];
 #pragma unroll
     for (int q = 0; q < kBatch; ++q) {
       const bool live = key[q] != PRESTO_NGRAM3_EMPTY;
-      kv[q] = live ? __ldg(a.keys + h[q]) : PRESTO_NGRAM3_EMPTY;
-      vv[q] = live ? __ldg(a.logrho + h[q]) : 0.f;
+      k0[q] = live ? __ldg(a.keys + h[q]) : PRESTO_NGRAM3_EMPTY;
+      v0[q] = live ? __ldg(a.logrho + h[q]) : 0.f;
+    }
+    // second round: the window after the home slot, for the probes still open
+    uint64_t kw[kBatch][kWin];
+    float vw[kBatch][kWin];
+#pragma unroll
+    for (int q = 0; q < kBatch; ++q) {
+      const bool open = k0[q] != key[q] && k0[q] != PRESTO_NGRAM3_EMPTY;
+#pragma unroll
+      for (int w = 0; w < kWin; ++w) {
+        const uint32_t hw = (h[q] + 1 + w) & a.cap_mask;
+        kw[q][w] = open ? __ldg(a.keys + hw) : PRESTO_NGRAM3_EMPTY;
+        vw[q][w] = open ? __ldg(a.logrho + hw) : 0.f;
+      }
     }
 #pragma unroll
     for (int q = 0; q < kBatch; ++q) {
@@ -432,13 +469,26 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
       if (f >= my) continue;
       float sc = lq[q];  // marginal-only: s = log q
       if (key[q] != PRESTO_NGRAM3_EMPTY) {
-        float lr;
-        if (kv[q] == key[q])
-          lr = vv[q];
-        else if (kv[q] == PRESTO_NGRAM3_EMPTY)
-          lr = a.miss;
-        else  // collision: continue the linear probe from the next slot
-          lr = probe_from(a.keys, a.logrho, a.cap_mask, a.miss, key[q], (h[q] + 1) & a.cap_mask);
+        // the first slot along the probe holding the key (a hit) or empty (a miss)
+        float lr = a.miss;
+        bool done = true;
+        if (k0[q] == key[q]) {
+          lr = v0[q];
+        } else if (k0[q] != PRESTO_NGRAM3_EMPTY) {
+          done = false;
+#pragma unroll
+          for (int w = 0; w < kWin; ++w) {
+            if (!done && kw[q][w] == key[q]) {
+              lr = vw[q][w];
+              done = true;
+            } else if (!done && kw[q][w] == PRESTO_NGRAM3_EMPTY) {
+              done = true;
+            }
+          }
+        }
+        if (!done)  // a chain longer than the window: continue slot by slot
+          lr = probe_from(a.keys, a.logrho, a.cap_mask, a.miss, key[q],
+                          (h[q] + 1 + kWin) & a.cap_mask);
         sc = __fadd_rn(__fmul_rn(a.lambda, lr), lq[q]);
       }
       if (sc > 0.f) report(a.dev_status, PRESTO_DEV_POSITIVE_SCORE);

@@ -6,19 +6,23 @@
 // dense contraction against that head's keys, so it runs on the 5th-generation
 // tensor cores, ping-ponging two 128-row tiles per CTA:
 //   * one CTA per (sequence, kv head, pair of 128-row tiles, KV split);
-//   * warp 8 loads both Q tiles, then K tiles of 64 keys into a 4-deep ring; warp 10
-//     loads V tiles into a 3-deep ring (TMA, 128-byte swizzle).  A K slot is refilled
-//     once both QK^T products of its tile completed, a V slot once both PV products
-//     did;
-//   * warp 9 issues tcgen05.mma: S_t = Q_t K^T (64 fp32 TMEM columns per row tile) one
-//     KV tile ahead of O_t += P_t V, where P_t (bf16) is read from TMEM.  The whole
-//     warp runs the issue loop and one elected lane issues, so descriptors stay on the
-//     uniform datapath;
+//   * warp 8 loads both Q tiles, then K tiles of 128 keys into a ring; warp 10 loads
+//     V tiles into another (TMA, 128-byte swizzle; 2 stages each at D = 128).  A K
+//     slot is refilled once both QK^T products of its tile completed, a V slot once
+//     both PV products did;
+//   * warp 9 issues tcgen05.mma: S_t = Q_t K^T (128 fp32 TMEM columns per row tile)
+//     and O_t += P_t V with P_t (bf16) read from TMEM, where the softmax wrote it over
+//     S_t.  Per KV tile: PV(t0), QK^T(t0) of the next tile, PV(t1), QK^T(t1); each
+//     QK^T waits for the completion of the PV that read the same TMEM, and the two
+//     row tiles ping-pong so that one tile's softmax overlaps the other tile's
+//     tensor work.  The whole warp runs the issue loop and one elected lane issues,
+//     so descriptors stay on the uniform datapath;
 //   * warps 0-3 and 4-7 run the softmax of tiles 0 and 1, one thread per query row
-//     (TMEM lane): tcgen05.ld of S, prefix-length and ancestor-bitmask masks (full
-//     prefix tiles skip them), online softmax with packed fp32x2 arithmetic, and
-//     tcgen05.st of P.  The running maximum is only moved (and O rescaled in TMEM)
-//     when it grows by more than 2^8, so most tiles skip the rescale;
+//     (TMEM lane): the row's 128 scores in registers (four tcgen05.ld in flight),
+//     prefix-length and ancestor-bitmask masks (full prefix tiles skip them), online
+//     softmax with packed fp32x2 arithmetic, P written back over S with tcgen05.st.
+//     The running maximum is only moved (and O rescaled in TMEM) when it grows by
+//     more than 2^8, so most tiles skip the rescale;
 //   * with several KV splits, the splits of one row block form a thread-block
 //     cluster (up to 16 CTAs): each CTA writes its rows' (m, l) and unnormalised fp32
 //     O to the workspace (column-quad-major, coalesced), the cluster synchronises
@@ -40,9 +44,7 @@ namespace presto {
 namespace {
 
 constexpr int kBM = 128;        // query rows per tile (TMEM lanes)
-constexpr int kBN = 64;         // keys per KV tile
-constexpr int kKStages = 4;     // K ring depth (K is needed two tiles before V)
-constexpr int kVStages = 3;     // V ring depth
+constexpr int kBN = 128;        // keys per KV tile
 // 11 warps: 0-3 and 4-7 run the softmax of row tiles 0 and 1 (one thread per query
 // row = TMEM lane), 8 loads Q and K, 9 issues tensor-core MMAs, 10 loads V
 constexpr int kThreads = 352;
@@ -54,10 +56,9 @@ constexpr float kRescaleLog2 = 8.f;  // move the running max only when it grows 
 constexpr int kRowBytes = 128;       // one 128-byte-swizzled row: 64 bf16
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
-// TMEM columns: S of tile t (64 fp32) at 64t, P of tile t (64 bf16 packed in pairs)
-// at 128 + 32t, O of tile t at 256 + 128t
+// TMEM columns: S of tile t (128 fp32) at 128t, overwritten in place by P of tile t
+// (128 bf16 packed in pairs, its first 64 columns); O of tile t at 256 + 128t
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kTmemP = 128;
 constexpr uint32_t kTmemO = 256;
 constexpr int kMaxSplits = 16;  // KV splits of a row block = CTAs of its cluster
 
@@ -75,13 +76,15 @@ struct Args {
 };
 
 // Shared memory: Q of both row tiles, the K ring, the V ring.  Every operand is
-// stored as 64-column panels of 128-byte rows with the 128-byte swizzle (Q: 128 rows
-// per panel, K and V: 64 rows per panel).
+// stored as 64-column panels of 128-byte rows with the 128-byte swizzle (128 rows
+// per panel).  Ring depths: 2 at D = 128 (192 KB in all), 4 at D = 64.
 template <int D>
 struct Layout {
+  static constexpr int kKStages = D == 64 ? 4 : 2;
+  static constexpr int kVStages = D == 64 ? 4 : 2;
   static constexpr int kPanels = D / 64;
   static constexpr int kQPanel = kBM * kRowBytes;   // 16 KB
-  static constexpr int kKVPanel = kBN * kRowBytes;  // 8 KB
+  static constexpr int kKVPanel = kBN * kRowBytes;  // 16 KB
   static constexpr int kQBytes = kBM * D * 2;
   static constexpr int kTileBytes = kBN * D * 2;    // one K or V tile
   static constexpr int kQ = 0;                          // tile 0, then tile 1
@@ -91,12 +94,12 @@ struct Layout {
   static constexpr int kAlloc = kBytes + 1024;  // room to align the base to 1024
 };
 
+constexpr int kMaxStages = 4;
 struct Bars {
   uint64_t q_full;
-  uint64_t k_full[kKStages], k_empty[kKStages];
-  uint64_t v_full[kVStages], v_empty[kVStages];
-  uint64_t s_full[2], s_free[2];
-  uint64_t p_full[2], o_done[2];
+  uint64_t k_full[kMaxStages], k_empty[kMaxStages];
+  uint64_t v_full[kMaxStages], v_empty[kMaxStages];
+  uint64_t s_full[2], p_full[2], o_done[2];
 };
 
 // Packed fp32 pairs (f32x2 arithmetic issues one instruction per two values) and
@@ -125,16 +128,15 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
   return d;
 }
 
-// One row's 64 scores of a KV tile -> the tile's row maximum (raw scores), as
-// eight independent three-input-max chains.
-__device__ __forceinline__ float row_max64(const float* v) {
-  float q[8];
+// 32 scores of a row -> their maximum, as four independent three-input-max chains.
+__device__ __forceinline__ float row_max32(const float* v) {
+  float q[4];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
+  for (int i = 0; i < 4; ++i) {
     const float* w = v + 8 * i;
     q[i] = fmaxf(max3(max3(max3(w[0], w[1], w[2]), w[3], w[4]), w[5], w[6]), w[7]);
   }
-  return max3(max3(q[0], q[1], q[2]), max3(q[3], q[4], q[5]), fmaxf(q[6], q[7]));
+  return max3(q[0], q[1], fmaxf(q[2], q[3]));
 }
 
 template <int D>
@@ -168,17 +170,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (tid == 0) {
     mbar_init(&bars.q_full, 1);
-    for (int st = 0; st < kKStages; ++st) {
+    for (int st = 0; st < kMaxStages; ++st) {
       mbar_init(&bars.k_full[st], 1);
       mbar_init(&bars.k_empty[st], 1);
-    }
-    for (int st = 0; st < kVStages; ++st) {
       mbar_init(&bars.v_full[st], 1);
       mbar_init(&bars.v_empty[st], 1);
     }
     for (int t = 0; t < 2; ++t) {
       mbar_init(&bars.s_full[t], 1);
-      mbar_init(&bars.s_free[t], kSoftThreads);
       mbar_init(&bars.p_full[t], kSoftThreads);
       mbar_init(&bars.o_done[t], 1);
     }
@@ -226,10 +225,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int p = 0; p < Ly::kPanels; ++p)
           tma_load_3d(smem + Ly::kQ + t * Ly::kQBytes + p * Ly::kQPanel, &tm_q, p * 64, g * a.G,
                       b * a.N + (mt0 + t) * nodes_per_tile, &bars.q_full);
-      // K_j -> slot j % kKStages, once both QK^T of K_{j - kKStages} completed
+      // K_j -> slot j % Ly::kKStages, once both QK^T of K_{j - Ly::kKStages} completed
       for (int j = 0; j < nt; ++j) {
-        const int st = j % kKStages;
-        if (j >= kKStages && !mbar_wait(&bars.k_empty[st], (j / kKStages - 1) & 1, abort)) {
+        const int st = j % Ly::kKStages;
+        if (j >= Ly::kKStages && !mbar_wait(&bars.k_empty[st], (j / Ly::kKStages - 1) & 1, abort)) {
           fail();
           break;
         }
@@ -250,10 +249,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       prefetch_tensormap(&tm_vc);
       prefetch_tensormap(&tm_vt);
-      // V_j -> slot j % kVStages, once both PV of V_{j - kVStages} completed
+      // V_j -> slot j % Ly::kVStages, once both PV of V_{j - Ly::kVStages} completed
       for (int j = 0; j < nt; ++j) {
-        const int st = j % kVStages;
-        if (j >= kVStages && !mbar_wait(&bars.v_empty[st], (j / kVStages - 1) & 1, abort)) {
+        const int st = j % Ly::kVStages;
+        if (j >= Ly::kVStages && !mbar_wait(&bars.v_empty[st], (j / Ly::kVStages - 1) & 1, abort)) {
           fail();
           break;
         }
@@ -271,10 +270,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (nt > 0 && warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
-    // QK^T runs one KV tile ahead of PV: for j: QK_{j+1}(t0), QK_{j+1}(t1) (each once
-    // that tile's softmax has read S_j), PV_j(t0), PV_j(t1) (P_j from TMEM).
-    // The whole warp runs this loop (wait outcomes made warp-uniform); one elected
-    // lane issues each MMA and commit.
+    // Per KV tile j and row tile t: PV_j(t) (P_t read from TMEM, where it overwrote
+    // S_t), then QK_{j+1}(t) into the same TMEM, issued once PV_j(t) has completed
+    // (its o_done), so S_t is never rewritten while P_t is still being read.  The whole warp runs this loop (wait outcomes made
+    // warp-uniform); one elected lane issues each MMA and commit.
     constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, false);
     constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, true);
     const uint64_t q_desc0 = smem_desc_sw128(smem_u32(smem + Ly::kQ), 16, 1024);
@@ -287,41 +286,55 @@ __global__ void __launch_bounds__(kThreads, 1)
     };
     // S_t = Q_t K_j^T
     auto qk = [&](int t, int j) {
-      if (j >= 1 && !wait(&bars.s_free[t], (j - 1) & 1)) return false;
       // descriptor start addresses are in 16-byte units in the low bits
       const uint64_t qd = q_desc0 + ((t * Ly::kQBytes) >> 4);
-      const uint64_t kd = k_desc0 + (((j % kKStages) * Ly::kTileBytes) >> 4);
+      const uint64_t kd = k_desc0 + (((j % Ly::kKStages) * Ly::kTileBytes) >> 4);
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t qo = ((kk >> 2) * Ly::kQPanel + (kk & 3) * 32) >> 4;
         const uint32_t ko = ((kk >> 2) * Ly::kKVPanel + (kk & 3) * 32) >> 4;
-        mma_bf16_warp(tmem_base + t * 64, qd + qo, kd + ko, idesc_qk, kk > 0);
+        mma_bf16_warp(tmem_base + t * 128, qd + qo, kd + ko, idesc_qk, kk > 0);
       }
       mma_commit_warp(&bars.s_full[t]);
-      return true;
     };
     // O_t (+)= P_t V_j, P_t read from TMEM (8 columns = 16 keys per step)
     auto pv = [&](int t, int j) {
       if (!wait(&bars.p_full[t], j & 1)) return false;
-      const uint64_t vd = v_desc0 + (((j % kVStages) * Ly::kTileBytes) >> 4);
+      const uint64_t vd = v_desc0 + (((j % Ly::kVStages) * Ly::kTileBytes) >> 4);
 #pragma unroll
       for (int kk = 0; kk < kBN / 16; ++kk)
-        mma_bf16_ts_warp(tmem_base + kTmemO + t * 128, tmem_base + kTmemP + t * 32 + kk * 8,
+        mma_bf16_ts_warp(tmem_base + kTmemO + t * 128, tmem_base + t * 128 + kk * 8,
                          vd + ((kk * 16 * kRowBytes) >> 4), idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
       mma_commit_warp(&bars.o_done[t]);
       return true;
     };
-    bool ok = wait(&bars.q_full, 0) && wait(&bars.k_full[0], 0) && qk(0, 0) && (!has1 || qk(1, 0));
-    if (ok) mma_commit_warp(&bars.k_empty[0]);
+    bool ok = wait(&bars.q_full, 0) && wait(&bars.k_full[0], 0);
+    if (ok) {
+      qk(0, 0);
+      if (has1) qk(1, 0);
+      mma_commit_warp(&bars.k_empty[0]);
+    }
+    // ping-pong: tile 0's next S is issued right after its PV, so its softmax runs
+    // while the tensor core works on tile 1, and the other way round
     for (int j = 0; ok && j < nt; ++j) {
-      if (j + 1 < nt) {
-        ok = wait(&bars.k_full[(j + 1) % kKStages], ((j + 1) / kKStages) & 1) && qk(0, j + 1) &&
-             (!has1 || qk(1, j + 1));
-        if (!ok) break;
-        mma_commit_warp(&bars.k_empty[(j + 1) % kKStages]);
+      const int jn = j + 1;
+      const bool more = jn < nt;
+      ok = wait(&bars.v_full[j % Ly::kVStages], (j / Ly::kVStages) & 1) && pv(0, j);
+      if (ok && more) {
+        ok = wait(&bars.k_full[jn % Ly::kKStages], (jn / Ly::kKStages) & 1) &&
+             wait(&bars.o_done[0], j & 1);
+        if (ok) qk(0, jn);
       }
-      ok = wait(&bars.v_full[j % kVStages], (j / kVStages) & 1) && pv(0, j) && (!has1 || pv(1, j));
-      if (ok) mma_commit_warp(&bars.v_empty[j % kVStages]);
+      if (ok && has1) {
+        ok = pv(1, j);
+        if (ok && more) {
+          ok = wait(&bars.o_done[1], j & 1);
+          if (ok) qk(1, jn);
+        }
+      }
+      if (!ok) break;
+      mma_commit_warp(&bars.v_empty[j % Ly::kVStages]);
+      if (more) mma_commit_warp(&bars.k_empty[jn % Ly::kKStages]);
     }
     if (!ok && lane == 0) fail();
   } else if (nt > 0 && warp < 4 * ntiles) {
@@ -331,7 +344,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = quad * 32 + lane;   // row of the tile
     const uint32_t lane_addr = static_cast<uint32_t>(quad * 32) << 16;
     const uint32_t tO = tmem_base + kTmemO + t * 128 + lane_addr;
-    const uint32_t tP = tmem_base + kTmemP + t * 32 + lane_addr;
+    const uint32_t tS = tmem_base + t * 128 + lane_addr;  // S_t, then P_t in place
     const int node = (mt0 + t) * nodes_per_tile + r / a.G;
     const int hh = r % a.G;
     const uint32_t* mrow =
@@ -339,78 +352,67 @@ __global__ void __launch_bounds__(kThreads, 1)
     float m = -INFINITY, l = 0.f;  // m: running (possibly stale) max, log2 domain
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
-      // wait outcomes are made warp-uniform: tcgen05.ld needs the whole warp
+      // wait outcomes are made warp-uniform: tcgen05.ld needs the whole warp.  S_j
+      // ready also means PV_{j-1} of this tile completed (QK_j was issued after it),
+      // so O_t may be rescaled and P_t rewritten.
       if (!__all_sync(0xffffffffu, mbar_wait(&bars.s_full[t], j & 1, abort))) {
         ok = false;
         break;
       }
       tc_fence_after();
-      float v[64];
-      const uint32_t tS = tmem_base + t * 64 + lane_addr;
-      tmem_ld32(tS, *reinterpret_cast<float(*)[32]>(v));
-      tmem_ld32(tS + 32, *reinterpret_cast<float(*)[32]>(v + 32));
-      // masks: prefix keys beyond kv_len; tree keys outside the ancestor set (a
-      // full prefix tile needs none)
-      uint32_t b0, b1;
+      // masks of the four 32-key chunks: prefix keys beyond kv_len; tree keys outside
+      // the ancestor set (a full prefix tile needs none)
+      uint32_t bits[4];
+      const bool full = j < n_prefix && kv - (t_begin + j) * kBN >= kBN;  // warp-uniform
       if (j < n_prefix) {
         const int lim = kv - (t_begin + j) * kBN;
-        b0 = lim >= 32 ? 0xffffffffu : (lim <= 0 ? 0u : (1u << lim) - 1u);
-        b1 = lim >= 64 ? 0xffffffffu : (lim <= 32 ? 0u : (1u << (lim - 32)) - 1u);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const int lc = lim - 32 * c;
+          bits[c] = lc >= 32 ? 0xffffffffu : (lc <= 0 ? 0u : (1u << lc) - 1u);
+        }
       } else {
         const int wi = ((j - n_prefix) * kBN) >> 5;
-        b0 = (mrow && wi < a.W) ? __ldg(mrow + wi) : 0u;
-        b1 = (mrow && wi + 1 < a.W) ? __ldg(mrow + wi + 1) : 0u;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) bits[c] = (mrow && wi + c < a.W) ? __ldg(mrow + wi + c) : 0u;
       }
-      const bool full = j < n_prefix && kv - (t_begin + j) * kBN >= kBN;  // warp-uniform
+      // the row's 128 scores: four loads in flight, one wait
+      float v[128];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, *reinterpret_cast<float(*)[32]>(v + 32 * c));
       tmem_wait_ld();
-      tc_fence_before();
-      mbar_arrive(&bars.s_free[t]);  // S_t may be overwritten by QK_{j+1}
       if (!full) {  // masked scores -> -inf (exp2 of -inf is 0)
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          v[e] = ((b0 >> e) & 1u) ? v[e] : -INFINITY;
-          v[32 + e] = ((b1 >> e) & 1u) ? v[32 + e] : -INFINITY;
-        }
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int e = 0; e < 32; ++e) v[32 * c + e] = ((bits[c] >> e) & 1u) ? v[32 * c + e] : -INFINITY;
       }
-      const float mx = row_max64(v) * a.scale_log2;  // scale > 0 commutes with max
+      float mx = fmaxf(fmaxf(row_max32(v), row_max32(v + 32)), fmaxf(row_max32(v + 64), row_max32(v + 96)));
+      mx *= a.scale_log2;  // scale > 0 commutes with max
       // stale-max online softmax: move m only when the row max exceeds it by > 2^8
       const bool move = mx > m + kRescaleLog2;
       const float alpha = move ? ex2(m - mx) : 1.f;
       if (move) m = mx;
       const float m_use = m == -INFINITY ? 0.f : m;
-      // p = exp2(s * scale - m); the row sum in four independent packed chains
+      // p = exp2(s * scale - m), stored as bf16 pairs over the S columns (P covers the
+      // first 64, all of S having been read); the row sum in packed chains
       const uint64_t sc2 = pack2(a.scale_log2, a.scale_log2), nm2 = pack2(-m_use, -m_use);
-      uint64_t acc[4] = {0ull, 0ull, 0ull, 0ull};
+      uint64_t acc[2] = {0ull, 0ull};
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        float x0, x1;
-        unpack2(fma2(pack2(v[2 * i], v[2 * i + 1]), sc2, nm2), x0, x1);
-        v[2 * i] = ex2(x0);
-        v[2 * i + 1] = ex2(x1);
-        acc[i & 3] = add2(acc[i & 3], pack2(v[2 * i], v[2 * i + 1]));
-      }
-      float rs, rs1;
-      unpack2(add2(add2(acc[0], acc[1]), add2(acc[2], acc[3])), rs, rs1);
-      rs += rs1;
-      l = l * alpha + rs;
-      if (j > 0) {  // P_t and O_t are free once PV_{j-1} of this tile completed
-        if (!__all_sync(0xffffffffu, mbar_wait(&bars.o_done[t], (j - 1) & 1, abort))) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-      }
-      // row r of P_t (64 keys as 32 bf16 pairs) into this thread's TMEM lane
-      {
-        uint32_t pk[32];
+      for (int c = 0; c < 4; ++c) {
+        uint32_t pk[16];
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          const __nv_bfloat162 pv2 = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
-          pk[e] = *reinterpret_cast<const uint32_t*>(&pv2);
+        for (int i = 0; i < 16; ++i) {
+          float x0, x1;
+          unpack2(fma2(pack2(v[32 * c + 2 * i], v[32 * c + 2 * i + 1]), sc2, nm2), x0, x1);
+          const float p0 = ex2(x0), p1 = ex2(x1);
+          acc[i & 1] = add2(acc[i & 1], pack2(p0, p1));
+          const __nv_bfloat162 pv2 = __floats2bfloat162_rn(p0, p1);
+          pk[i] = *reinterpret_cast<const uint32_t*>(&pv2);
         }
-        tmem_st32(tP, *reinterpret_cast<const float(*)[32]>(pk));
+        tmem_st16(tS + c * 16, pk);
       }
-      if (j > 0 && __any_sync(0xffffffffu, move)) {
+      if (j > 0 && __any_sync(0xffffffffu, move)) {  // O_t *= alpha (rows that did not move: 1)
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
@@ -421,6 +423,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_st32(tO + c * 32, o);
         }
       }
+      float rs, rs1;
+      unpack2(add2(acc[0], acc[1]), rs, rs1);
+      l = l * alpha + (rs + rs1);
       tmem_wait_st();  // P (and a rescaled O) are in TMEM before the MMA is released
       tc_fence_before();
       mbar_arrive(&bars.p_full[t]);

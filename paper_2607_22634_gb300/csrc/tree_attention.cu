@@ -24,8 +24,8 @@
 //     The running maximum is only moved (and O rescaled in TMEM) when it grows by
 //     more than 2^8, so most tiles skip the rescale;
 //   * with several KV splits, the splits of one row block form a thread-block
-//     cluster (up to 16 CTAs): each CTA writes its rows' (m, l) and unnormalised fp32
-//     O to the workspace (column-quad-major, coalesced), the cluster synchronises
+//     cluster (up to 16 CTAs): each CTA writes its rows' fp32 (m, l) and O / l as
+//     bf16 to the workspace (column-quad-major, coalesced), the cluster synchronises
 //     (release / acquire), and each CTA merges a slice of the rows over the splits
 //     with log-sum-exp weights, all loads of a row issued together.
 // Every wait is bounded; on time-out the CTA records PRESTO_DEV_TIMEOUT and unwinds.
@@ -70,7 +70,7 @@ struct Args {
   float scale_log2;
   __nv_bfloat16* out;
   float* lse;
-  float4* part_o;   // KV splits: unnormalised fp32 O [CTA][D / 4][2 * kBM] (column quads)
+  uint2* part_o;    // KV splits: O / l of each row as bf16 [CTA][D / 4][2 * kBM] (column quads)
   float2* part_ml;  // KV splits: (m, l) per row [CTA][2 * kBM], log2 domain
   int32_t* dev_status;
 };
@@ -152,6 +152,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ Bars bars;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
+  __shared__ float mw[kBM][kMaxSplits + 1];  // split merge: per-row weights (slice <= kBM rows)
+  __shared__ float mlse[kBM];                // split merge: per-row lse
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   int idx = blockIdx.x;
@@ -440,16 +442,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       a.part_ml[prow] = ok ? make_float2(m, l) : make_float2(-INFINITY, 0.f);
       if (ok) {
         tc_fence_after();
-        // column-quad-major, so a warp's 32 rows of one quad are 512 contiguous bytes
-        float4* dst = a.part_o + static_cast<size_t>(blockIdx.x) * (D / 4) * 2 * kBM + t * kBM + r;
+        // the row normalised by its own l, as bf16 (values stay within the range of V),
+        // column-quad-major so that a warp's 32 rows of one quad are 256 contiguous bytes
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        uint2* dst = a.part_o + static_cast<size_t>(blockIdx.x) * (D / 4) * 2 * kBM + t * kBM + r;
 #pragma unroll 1
         for (int c = 0; c < D / 32; ++c) {
           float o[32];
           tmem_ld32(tO + c * 32, o);
           tmem_wait_ld();
 #pragma unroll
-          for (int q = 0; q < 8; ++q)
-            dst[(c * 8 + q) * 2 * kBM] = make_float4(o[q * 4], o[q * 4 + 1], o[q * 4 + 2], o[q * 4 + 3]);
+          for (int q = 0; q < 8; ++q) {
+            const __nv_bfloat162 lo = __floats2bfloat162_rn(o[q * 4] * inv, o[q * 4 + 1] * inv);
+            const __nv_bfloat162 hi = __floats2bfloat162_rn(o[q * 4 + 2] * inv, o[q * 4 + 3] * inv);
+            dst[(c * 8 + q) * 2 * kBM] = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
+                                                    *reinterpret_cast<const uint32_t*>(&hi));
+          }
         }
       }
     } else if (ok) {
@@ -526,52 +534,78 @@ __global__ void __launch_bounds__(kThreads, 1)
   const size_t cta0 = static_cast<size_t>(blockIdx.x - split);  // first CTA of the cluster
   const int r0 = split * slice;
   const int nr = max(0, min(R, r0 + slice) - r0);
-  constexpr int kC4 = D / 4;  // float4 columns per row
-  // one item = one row of the slice x one column quad; all its loads (every split's
-  // (m, l) and partial) are issued together, so the merge costs one L2 round trip
-  for (int item = tid; item < nr * kC4; item += kThreads) {
-    const int c4 = item / nr, i = item % nr;  // rows fastest: coalesced partial loads
-    const int row = r0 + i;
-    const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
-    const int hh = (row % kBM) % a.G;
-    if (node >= a.N) continue;
-    float2 ml[kMaxSplits];
-    float4 o[kMaxSplits];
+  constexpr int kC4 = D / 4;  // 4-column quads per row
+  // One item = one row of the slice x one column quad, rows fastest (coalesced
+  // partial loads).  Each thread's first two items are loaded before the per-row
+  // weights are formed (one thread per row, into shared memory), so the usual case
+  // costs one L2 round trip.
+  const int nitems = nr * kC4;
+  auto load_item = [&](int item, uint2 (&o)[kMaxSplits]) {
+    const int c4 = item / nr, row = r0 + item % nr;
 #pragma unroll
-    for (int s = 0; s < kMaxSplits; ++s) {
-      const bool in = s < nsp;
-      ml[s] = in ? __ldcg(a.part_ml + (cta0 + s) * 2 * kBM + row) : make_float2(-INFINITY, 0.f);
-      o[s] = in ? __ldcg(a.part_o + ((cta0 + s) * kC4 + c4) * 2 * kBM + row)
-                : make_float4(0.f, 0.f, 0.f, 0.f);
-    }
+    for (int s = 0; s < kMaxSplits; ++s)
+      o[s] = (item < nitems && s < nsp)
+                 ? __ldcg(a.part_o + ((cta0 + s) * kC4 + c4) * 2 * kBM + row)
+                 : make_uint2(0u, 0u);
+  };
+  uint2 oa[kMaxSplits], ob[kMaxSplits];
+  load_item(tid, oa);
+  load_item(tid + kThreads, ob);
+  if (tid < nr) {
+    // the row's weights over the splits, w_s l_s / L (a split without keys for the row
+    // has m = -inf and weight 0), and its lse
+    const int row = r0 + tid;
+    float2 ml[kMaxSplits];
+#pragma unroll
+    for (int s = 0; s < kMaxSplits; ++s)
+      ml[s] = s < nsp ? __ldcg(a.part_ml + (cta0 + s) * 2 * kBM + row) : make_float2(-INFINITY, 0.f);
     float M = -INFINITY;
 #pragma unroll
     for (int s = 0; s < kMaxSplits; ++s) M = fmaxf(M, ml[s].x);
-    float L = 0.f;
+    float wl[kMaxSplits], L = 0.f;
+#pragma unroll
+    for (int s = 0; s < kMaxSplits; ++s) {
+      wl[s] = (M == -INFINITY || ml[s].x == -INFINITY) ? 0.f : ex2(ml[s].x - M) * ml[s].y;
+      L += wl[s];
+    }
+    const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
+    const bool used = node < nn && L > 0.f;
+    const float inv = used ? 1.f / L : 0.f;
+#pragma unroll
+    for (int s = 0; s < kMaxSplits; ++s) mw[tid][s] = wl[s] * inv;
+    mlse[tid] = used ? (M + log2f(L)) * kLn2 : -INFINITY;
+  }
+  __syncthreads();
+  auto finish_item = [&](int item, const uint2 (&o)[kMaxSplits]) {
+    if (item >= nitems) return;
+    const int c4 = item / nr, i = item % nr;
+    const int row = r0 + i;
+    const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
+    const int hh = (row % kBM) % a.G;
+    if (node >= a.N) return;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
     for (int s = 0; s < kMaxSplits; ++s) {
-      // a split without keys for the row (m = -inf) wrote no O: weight 0, value unused
-      if (M == -INFINITY || ml[s].x == -INFINITY) continue;
-      const float w = ex2(ml[s].x - M);
-      L += ml[s].y * w;
-      acc.x += w * o[s].x;
-      acc.y += w * o[s].y;
-      acc.z += w * o[s].z;
-      acc.w += w * o[s].w;
+      const float w = mw[i][s];  // 0 for absent splits: their (zero) values are unused
+      acc.x += w * __uint_as_float(o[s].x << 16);
+      acc.y += w * __uint_as_float(o[s].x & 0xffff0000u);
+      acc.z += w * __uint_as_float(o[s].y << 16);
+      acc.w += w * __uint_as_float(o[s].y & 0xffff0000u);
     }
-    const bool used = node < nn && L > 0.f;
-    const float inv = used ? 1.f / L : 0.f;
     const size_t orow = ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
-    const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-    const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
+    const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
     uint2 u2;
     u2.x = *reinterpret_cast<const uint32_t*>(&lo);
     u2.y = *reinterpret_cast<const uint32_t*>(&hi);
     *reinterpret_cast<uint2*>(a.out + orow + c4 * 4) = u2;
-    if (c4 == 0 && a.lse)
-      a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] =
-          used ? (M + log2f(L)) * kLn2 : -INFINITY;
+    if (c4 == 0 && a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = mlse[i];
+  };
+  finish_item(tid, oa);
+  finish_item(tid + kThreads, ob);
+  for (int item = tid + 2 * kThreads; item < nitems; item += kThreads) {
+    load_item(item, oa);
+    finish_item(item, oa);
   }
 }
 
@@ -704,11 +738,11 @@ using namespace presto;
 extern "C" size_t presto_attn_workspace(int B, int N, int Hq, int Hkv, int D, int Tmax) {
   if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || Tmax < 1 || (D != 64 && D != 128))
     return 0;
-  // KV splits leave fp32 partial rows and (m, l) for the in-kernel merge
+  // KV splits leave bf16 partial rows and fp32 (m, l) for the in-kernel merge
   const int* active = D == 128 ? active_clusters<128>() : active_clusters<64>();
   const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
   if (p.n_splits == 1) return 256;
-  return align_up(p.ctas * 2 * kBM * (static_cast<size_t>(D) * 4 + 8), 256);
+  return align_up(p.ctas * 2 * kBM * (static_cast<size_t>(D) * 2 + 8), 256);
 }
 
 extern "C" int presto_tree_attention(const void* q, const void* k_cache, const void* v_cache,
@@ -732,10 +766,10 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
   const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
   Args a{};
   if (p.n_splits > 1) {
-    const size_t need = p.ctas * 2 * kBM * (static_cast<size_t>(D) * 4 + 8);
+    const size_t need = p.ctas * 2 * kBM * (static_cast<size_t>(D) * 2 + 8);
     if (!ws || reinterpret_cast<uintptr_t>(ws) % 16 || ws_bytes < need) return PRESTO_ERR_WORKSPACE;
-    a.part_o = static_cast<float4*>(ws);
-    a.part_ml = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.ctas * 2 * kBM * D * 4);
+    a.part_o = static_cast<uint2*>(ws);
+    a.part_ml = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.ctas * 2 * kBM * D * 2);
   }
   const uint64_t e = 2;  // bf16 bytes
   CUtensorMap tq, tkc, tvc, tkt, tvt;

@@ -30,14 +30,16 @@ R7  Best-first (Alg. 2) commits a node when it is popped from the frontier
     exactly the top-N prefix-closed set of §4.2 ("the optimal tree consists of
     the B prefixes with the largest S").  Alg. 2 as printed adds all b children
     to the tree at expansion time, which can keep a shallow low-score child over
-    a deeper high-score one; ``eager_best_first_tree`` keeps that variant for
-    comparison only.
+    a deeper high-score one; ``eager_tree`` computes that variant.
 R8  Tree attention: softmax(scale * q k^T) v over every committed prefix key plus
     the tree keys that are ancestors-or-self of the query node; scale = 1/sqrt(D)
     unless given; no soft-cap; rows of unused node slots are zero with lse = -inf.
 R9  Acceptance (§2.1, App. A alpha_T(P)): the deepest node whose root path is
     the target's greedy continuation; the bonus token is the target's token after
     that node.
+R10 Beam search (Alg. 1): TopW and TopB use the total order R6; the loop runs
+    while |T| < N, counting every node added to T (root included); a depth whose
+    beam is empty ends the search.
 """
 
 from __future__ import annotations
@@ -188,29 +190,107 @@ def best_first_tree(ids, logq, ctx, table, miss, lam, bfac, N, precision="fp32")
     return out
 
 
-def eager_best_first_tree(ids, logq, ctx, table, miss, lam, bfac, N, precision="fp64"):
-    """Alg. 2 exactly as printed: children join T when their parent is expanded;
-    the loop stops once |T| >= N and TopB(T, N) is returned.  Kept only to show
-    where it departs from the lazy reading R7 (it is not the method's output)."""
+class _Nodes:
+    """Nodes of one sequence's search tree: node 0 is the root.  Each node keeps
+    its root path, S in the search precision, S recomputed in float64, the rank of
+    its token among the position's top-k, its depth and its parent."""
+
+    def __init__(self, ctx2):
+        self.path, self.S, self.S64, self.rank, self.parent = [()], [0.0], [0.0], [-1], [-1]
+        self.root_token = int(ctx2[1])
+        self._key = {}
+
+    def add(self, parent, t, S, s64, j):
+        self.path.append(self.path[parent] + (t,))
+        self.S.append(S)
+        self.S64.append(self.S64[parent] + s64)
+        self.rank.append(j)
+        self.parent.append(parent)
+        return len(self.path) - 1
+
+    def key(self, v):
+        """The total order R6 without output indices: (-S, depth, token, key(parent)),
+        compared lexicographically; the root's key () sorts first."""
+        if v not in self._key:
+            p = self.path[v]
+            self._key[v] = () if not p else (-float(self.S[v]), len(p), p[-1],
+                                            self.key(self.parent[v]))
+        return self._key[v]
+
+    def expand(self, v, ids_b, logq_b, ctx2, table, miss, lam, bfac, precision):
+        """§4.2 expansion: add the top-b children of v (R5); returns their node ids."""
+        p = self.path[v]
+        if len(p) >= ids_b.shape[0]:
+            return []
+        a, bb = trigram_context(ctx2, p)
+        out = []
+        for s, t, j in children(ids_b, logq_b, ctx2, table, miss, lam, bfac, p, precision):
+            rho = None if table is None else table.get((a, bb, t), miss)
+            s64 = token_score(logq_b[len(p), j], rho, lam, "fp64")
+            out.append(self.add(v, t, path_add(self.S[v], s, precision), s64, j))
+        return out
+
+    def write(self, out, b, chosen):
+        """Write the chosen node ids, sorted by the total order, as output rows."""
+        order = sorted(chosen, key=self.key)
+        index = {v: i for i, v in enumerate(order)}
+        for i, v in enumerate(order):
+            if v and self.parent[v] not in index:
+                raise AssertionError("selected set is not prefix-closed")
+            out["token"][b, i] = self.root_token if v == 0 else self.path[v][-1]
+            out["parent"][b, i] = -1 if v == 0 else index[self.parent[v]]
+            out["depth"][b, i] = len(self.path[v])
+            out["score"][b, i] = float(self.S[v])
+            out["score64"][b, i] = self.S64[v]
+            out["rank"][b, i] = self.rank[v]
+        out["n_nodes"][b] = len(order)
+
+
+def beam_search_tree(ids, logq, ctx, table, miss, lam, bfac, N, W, precision="fp32"):
+    """Beam search with global retention (§4.2, Alg. 1).
+
+    P = {root}, T = {root}.  For depth d = 1..L, while |T| < N: every node of the
+    beam P is expanded by its top-b children (§4.2 expansion step 2); all of them
+    join T, and the W best of them (total order R6) become the next beam.  The
+    result is TopB(T, N): the N best nodes of T in the order R6.  Same output arrays
+    as best_first_tree.
+    """
     ids = np.asarray(ids)
     logq = np.asarray(logq, dtype=np.float64)
     B, L, _ = ids.shape
-    result = []
+    out = _empty_tree(B, N)
     for b in range(B):
-        nodes = [(0.0, 0, int(ctx[b][1]), ())]        # (S, depth, token, path)
-        frontier = [(-0.0, 0, 0)]                      # (-S, depth, node index)
-        while len(nodes) < N and frontier:
-            _, _, v = heapq.heappop(frontier)
-            Sv, dv, _, pv = nodes[v]
-            if dv >= L:
-                continue
-            for s, t, _ in children(ids[b], logq[b], ctx[b], table, miss, lam, bfac,
-                                    pv, precision):
-                nodes.append((path_add(Sv, s, precision), dv + 1, t, pv + (t,)))
-                heapq.heappush(frontier, (-nodes[-1][0], dv + 1, len(nodes) - 1))
-        nodes.sort(key=lambda e: (-e[0], e[1], e[2]))
-        result.append(sorted(e[3] for e in nodes[:N]))
-    return result
+        T = _Nodes(ctx[b])
+        P = [0]
+        for d in range(1, L + 1):
+            if len(T.path) >= N or not P:
+                break
+            P_new = []
+            for v in P:
+                P_new += T.expand(v, ids[b], logq[b], ctx[b], table, miss, lam, bfac, precision)
+            P = sorted(P_new, key=T.key)[:W]
+        T.write(out, b, sorted(range(len(T.path)), key=T.key)[:N])
+    return out
+
+
+def eager_tree(ids, logq, ctx, table, miss, lam, bfac, N, precision="fp32"):
+    """Alg. 2 exactly as printed (the eager variant of R7): P = {root}, T = {root};
+    while |T| < N, pop the best node of P (order R6), expand it, and add its
+    children to both P and T; return TopB(T, N).  Same output arrays as
+    best_first_tree."""
+    ids = np.asarray(ids)
+    logq = np.asarray(logq, dtype=np.float64)
+    B, L, _ = ids.shape
+    out = _empty_tree(B, N)
+    for b in range(B):
+        T = _Nodes(ctx[b])
+        P = [(T.key(0), 0)]
+        while len(T.path) < N and P:
+            _, v = heapq.heappop(P)
+            for c in T.expand(v, ids[b], logq[b], ctx[b], table, miss, lam, bfac, precision):
+                heapq.heappush(P, (T.key(c), c))
+        T.write(out, b, sorted(range(len(T.path)), key=T.key)[:N])
+    return out
 
 
 def candidate_tree_nodes(ids_b, logq_b, ctx2, table, miss, lam, bfac, precision):

@@ -72,8 +72,8 @@ def test_lazy_reading_beats_printed_eager_variant():
     ids, logq, ctx, (A, B, C, D, E, F) = _lazy_vs_eager_case()
     lazy = O.best_first_tree(ids, logq, ctx, None, 0.0, 0.0, 2, 4, "fp64")
     assert lazy["token"][0].tolist() == [1, A, C, E]
-    eager = O.eager_best_first_tree(ids, logq, ctx, None, 0.0, 0.0, 2, 4)[0]
-    assert eager == sorted([(), (A,), (A, C), (B,)])
+    eager = O.eager_tree(ids, logq, ctx, None, 0.0, 0.0, 2, 4, "fp64")
+    assert eager["token"][0].tolist() == [1, A, C, B]
     obj = lambda S: sum(math.exp(s) for s in S)          # Eq. surrogate-objective
     assert obj([0, -1, -1.1, -1.2]) > obj([0, -1, -1.1, -5])
 

@@ -6,6 +6,7 @@
  *
  *   presto_topk             per-position log-softmax and top-k of the drafter logits
  *   presto_score_build_tree prefix-aligned scores + best-first tree up to N nodes
+ *                           (_ex: beam search / printed Alg. 2, per-position lambda)
  *   presto_tree_mask        ancestor bitmask and position ids of the tree tokens
  *   presto_tree_attention   tree-masked GQA attention against the KV-cache prefix
  *   presto_accept           longest accepted root path under greedy verification
@@ -191,6 +192,41 @@ int presto_score_build_tree(const int32_t* topk_ids, const float* topk_logq, int
                             int32_t* node_depth, float* node_score, int32_t* n_nodes,
                             void* ws, size_t ws_bytes, int32_t* dev_status,
                             presto_stream_t stream);
+
+/*
+ * presto_score_build_tree_ex - presto_score_build_tree with a choice of search
+ * policy (§4.2) and of a per-position lambda.
+ *
+ *   lambda_d    nullable [B, L] float32 (device): lambda of each drafter row (row d-1
+ *               scores depth d), e.g. the entropy-adaptive lambda_d(H_d) of App. F
+ *               written by presto_topk_entropy; NULL uses `lambda` everywhere.
+ *               Values must be >= 0.
+ *   policy      PRESTO_SEARCH_BEST_FIRST: as presto_score_build_tree (Alg. 2 with a
+ *                 node committed when it is popped: the N best nodes of the
+ *                 candidate tree).
+ *               PRESTO_SEARCH_BEAM: beam search with global retention (Alg. 1): from
+ *                 the beam {root}, while the tree T holds fewer than N nodes, every
+ *                 beam node gains its top-b children (all join T) and the
+ *                 `beam_width` best of them form the next beam; the result is the
+ *                 N best nodes of T.  The paper's default (beam width 10, §5.1).
+ *               PRESTO_SEARCH_EAGER: Alg. 2 as printed: pop the best frontier node,
+ *                 add all its children to T, until |T| >= N; the N best nodes of T.
+ *   beam_width  >= 1 (used by PRESTO_SEARCH_BEAM; <= 256).
+ * "Best" is always the order S desc, depth asc, token asc, parent index asc, and
+ * the output is stored in that order (parent index < child index).
+ *   ws          presto_build_workspace_ex(B, L, k, N, beam_width) bytes.
+ */
+#define PRESTO_SEARCH_BEST_FIRST 0
+#define PRESTO_SEARCH_BEAM 1
+#define PRESTO_SEARCH_EAGER 2
+size_t presto_build_workspace_ex(int B, int L, int k, int N, int beam_width);
+int presto_score_build_tree_ex(const int32_t* topk_ids, const float* topk_logq, int B, int L,
+                               int k, int b, const int32_t* ctx2, const presto_ngram3* ngram,
+                               float lambda, const float* lambda_d, int policy, int beam_width,
+                               int N, int32_t* node_token, int32_t* node_parent,
+                               int32_t* node_depth, float* node_score, int32_t* n_nodes,
+                               void* ws, size_t ws_bytes, int32_t* dev_status,
+                               presto_stream_t stream);
 
 /*
  * presto_tree_mask - tree attention mask and position ids (§4.3 and App. C (I),

@@ -109,6 +109,17 @@ def path_add(S_parent, s, precision: str):
     return F32(F32(S_parent) + F32(s))                            # R4
 
 
+def _lam_of(lam, b):
+    """lambda of sequence b: a scalar for every row, or row b of a [B, L] array
+    (App. F: a lambda_d per position)."""
+    return lam[b] if np.ndim(lam) == 2 else lam
+
+
+def _lam_at(lam_b, row):
+    """lambda of drafter row `row` (depth row + 1)."""
+    return float(lam_b[row]) if np.ndim(lam_b) == 1 else lam_b
+
+
 def children(ids_b, logq_b, ctx2, table, miss, lam, bfac, path, precision):
     """Top-b children of the node with root path `path` (R5).
 
@@ -120,7 +131,7 @@ def children(ids_b, logq_b, ctx2, table, miss, lam, bfac, path, precision):
     for j in range(ids_b.shape[1]):
         t = int(ids_b[d, j])
         rho = None if table is None else table.get((a, bb, t), miss)
-        out.append((token_score(logq_b[d, j], rho, lam, precision), t, j))
+        out.append((token_score(logq_b[d, j], rho, _lam_at(lam, d), precision), t, j))
     out.sort(key=lambda e: (-float(e[0]), e[1]))
     return out[:bfac]
 
@@ -156,6 +167,7 @@ def best_first_tree(ids, logq, ctx, table, miss, lam, bfac, N, precision="fp32")
     B, L, _ = ids.shape
     out = _empty_tree(B, N)
     for b in range(B):
+        lam_b = _lam_of(lam, b)
         tok = [int(ctx[b][1])]
         par, dep, S, S64, rank, paths = [-1], [0], [0.0], [0.0], [-1], [()]
         frontier = []
@@ -163,7 +175,7 @@ def best_first_tree(ids, logq, ctx, table, miss, lam, bfac, N, precision="fp32")
         def expand(n):
             if dep[n] >= L:
                 return
-            for s, t, j in children(ids[b], logq[b], ctx[b], table, miss, lam, bfac,
+            for s, t, j in children(ids[b], logq[b], ctx[b], table, miss, lam_b, bfac,
                                     paths[n], precision):
                 Sc = path_add(S[n], s, precision)
                 # heapq pops the smallest tuple: the key order is R6.
@@ -176,7 +188,7 @@ def best_first_tree(ids, logq, ctx, table, miss, lam, bfac, N, precision="fp32")
             if table is not None:
                 rho = table.get(trigram_context(ctx[b], paths[p]) + (t,), miss)
             tok.append(t); par.append(p); dep.append(d); S.append(Sc); rank.append(j)
-            S64.append(S64[p] + token_score(logq[b, d - 1, j], rho, lam, "fp64"))
+            S64.append(S64[p] + token_score(logq[b, d - 1, j], rho, _lam_at(lam_b, d - 1), "fp64"))
             paths.append(paths[p] + (t,))
             expand(len(tok) - 1)
         n = len(tok)
@@ -226,7 +238,7 @@ class _Nodes:
         out = []
         for s, t, j in children(ids_b, logq_b, ctx2, table, miss, lam, bfac, p, precision):
             rho = None if table is None else table.get((a, bb, t), miss)
-            s64 = token_score(logq_b[len(p), j], rho, lam, "fp64")
+            s64 = token_score(logq_b[len(p), j], rho, _lam_at(lam, len(p)), "fp64")
             out.append(self.add(v, t, path_add(self.S[v], s, precision), s64, j))
         return out
 
@@ -267,7 +279,8 @@ def beam_search_tree(ids, logq, ctx, table, miss, lam, bfac, N, W, precision="fp
                 break
             P_new = []
             for v in P:
-                P_new += T.expand(v, ids[b], logq[b], ctx[b], table, miss, lam, bfac, precision)
+                P_new += T.expand(v, ids[b], logq[b], ctx[b], table, miss, _lam_of(lam, b), bfac,
+                                  precision)
             P = sorted(P_new, key=T.key)[:W]
         T.write(out, b, sorted(range(len(T.path)), key=T.key)[:N])
     return out
@@ -287,7 +300,8 @@ def eager_tree(ids, logq, ctx, table, miss, lam, bfac, N, precision="fp32"):
         P = [(T.key(0), 0)]
         while len(T.path) < N and P:
             _, v = heapq.heappop(P)
-            for c in T.expand(v, ids[b], logq[b], ctx[b], table, miss, lam, bfac, precision):
+            for c in T.expand(v, ids[b], logq[b], ctx[b], table, miss, _lam_of(lam, b), bfac,
+                              precision):
                 heapq.heappush(P, (T.key(c), c))
         T.write(out, b, sorted(range(len(T.path)), key=T.key)[:N])
     return out
@@ -310,7 +324,8 @@ def candidate_tree_nodes(ids_b, logq_b, ctx2, table, miss, lam, bfac, precision)
             for d in range(1, len(cpath) + 1):
                 a, bb = trigram_context(ctx2, cpath[: d - 1])
                 rho = None if table is None else table.get((a, bb, cpath[d - 1]), miss)
-                S = path_add(S, token_score(logq_b[d - 1, cranks[d - 1]], rho, lam, precision),
+                S = path_add(S, token_score(logq_b[d - 1, cranks[d - 1]], rho, _lam_at(lam, d - 1),
+                                            precision),
                              precision)
             nodes.append((cpath, S, cranks))
             stack.append((cpath, cranks))
@@ -331,7 +346,8 @@ def brute_force_tree(ids, logq, ctx, table, miss, lam, bfac, N, precision="fp32"
     B = ids.shape[0]
     out = _empty_tree(B, N)
     for b in range(B):
-        nodes = candidate_tree_nodes(ids[b], logq[b], ctx[b], table, miss, lam, bfac, precision)
+        nodes = candidate_tree_nodes(ids[b], logq[b], ctx[b], table, miss, _lam_of(lam, b), bfac,
+                                     precision)
         by_path = {e[0]: e for e in nodes}
         keys = {}
 

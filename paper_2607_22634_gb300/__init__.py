@@ -8,6 +8,9 @@ resident and replays the five calls (optionally as one CUDA graph).
 
 from ._lib import (  # noqa: F401
     DEV_STATUS_BITS,
+    SEARCH_BEAM,
+    SEARCH_BEST_FIRST,
+    SEARCH_EAGER,
     Ngram3Table,
     PrestoError,
     dev_status_names,

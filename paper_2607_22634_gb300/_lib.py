@@ -51,6 +51,10 @@ _SIGS = {
     "presto_ngram3_clear": (_I, [ctypes.POINTER(Ngram3), _P]),
     "presto_ngram3_insert": (_I, [ctypes.POINTER(Ngram3), _P, _P, _I, _P, _P]),
     "presto_build_workspace": (ctypes.c_size_t, [_I, _I, _I, _I]),
+    "presto_build_workspace_ex": (ctypes.c_size_t, [_I, _I, _I, _I, _I]),
+    "presto_score_build_tree_ex": (_I, [_P, _P, _I, _I, _I, _I, _P, ctypes.POINTER(Ngram3),
+                                        ctypes.c_float, _P, _I, _I, _I, _P, _P, _P, _P, _P,
+                                        _P, ctypes.c_size_t, _P, _P]),
     "presto_score_build_tree": (_I, [_P, _P, _I, _I, _I, _I, _P, ctypes.POINTER(Ngram3),
                                      ctypes.c_float, _I, _P, _P, _P, _P, _P, _P,
                                      ctypes.c_size_t, _P, _P]),
@@ -220,32 +224,41 @@ class Ngram3Table:
 
 # ------------------------------------------------------------------ tree build
 
-def presto_build_workspace(B, L, k, N) -> int:
-    return int(load().presto_build_workspace(B, L, k, N))
+SEARCH_BEST_FIRST, SEARCH_BEAM, SEARCH_EAGER = 0, 1, 2
+
+
+def presto_build_workspace(B, L, k, N, beam_width=1) -> int:
+    return int(load().presto_build_workspace_ex(B, L, k, N, beam_width))
 
 
 def presto_score_build_tree(topk_ids, topk_logq, ctx2, ngram, lam, N, b=None, out=None, ws=None,
-                            dev_status=None, stream=None):
-    """Returns dict(token, parent, depth, score, n_nodes) of device tensors."""
+                            dev_status=None, stream=None, lambda_d=None,
+                            policy=SEARCH_BEST_FIRST, beam_width=1):
+    """Returns dict(token, parent, depth, score, n_nodes) of device tensors.
+    ``lambda_d`` ([B, L] float32, optional) gives each drafter row its own lambda;
+    ``policy`` is SEARCH_BEST_FIRST, SEARCH_BEAM (with ``beam_width``) or SEARCH_EAGER."""
     B, L, k = topk_ids.shape
     b = k if b is None else b
     dev = topk_ids.device
     _need(topk_ids, torch.int32, (B, L, k), "topk_ids")
     _need(topk_logq, torch.float32, (B, L, k), "topk_logq")
     _need(ctx2, torch.int32, (B, 2), "ctx2")
+    if lambda_d is not None:
+        _need(lambda_d, torch.float32, (B, L), "lambda_d")
     if out is None:
         out = {"token": torch.empty(B, N, dtype=torch.int32, device=dev),
                "parent": torch.empty(B, N, dtype=torch.int32, device=dev),
                "depth": torch.empty(B, N, dtype=torch.int32, device=dev),
                "score": torch.empty(B, N, dtype=torch.float32, device=dev),
                "n_nodes": torch.empty(B, dtype=torch.int32, device=dev)}
-    ws, nws = _ws(presto_build_workspace(B, L, k, N), dev, ws)
+    ws, nws = _ws(presto_build_workspace(B, L, k, N, beam_width), dev, ws)
     desc = None if ngram is None else ctypes.byref(ngram.desc)
-    st = load().presto_score_build_tree(
-        _ptr(topk_ids), _ptr(topk_logq), B, L, k, b, _ptr(ctx2), desc, float(lam), N,
+    st = load().presto_score_build_tree_ex(
+        _ptr(topk_ids), _ptr(topk_logq), B, L, k, b, _ptr(ctx2), desc, float(lam),
+        _ptr(lambda_d), int(policy), int(beam_width), N,
         _ptr(out["token"]), _ptr(out["parent"]), _ptr(out["depth"]), _ptr(out["score"]),
         _ptr(out["n_nodes"]), _ptr(ws), nws, _ptr(dev_status), _stream(stream))
-    _check(st, "presto_score_build_tree")
+    _check(st, "presto_score_build_tree_ex")
     return out
 
 

@@ -80,6 +80,8 @@ struct Args {
   uint32_t cap_mask;
   float miss;
   float lambda;
+  const float* lambda_d;  // [B, L] per-row lambda, or null (use `lambda`)
+  int policy, W;          // PRESTO_SEARCH_*, beam width
   int use_table;
   int L, k, bf, N;
   int nctx_all;      // contexts of one sequence over all depths
@@ -107,6 +109,7 @@ struct Smem {
   int cid[kMaxL][kMaxK];          // candidate tokens of every depth
   float clq[kMaxL][kMaxK];        // their log q
   int ctx0, ctx1;
+  float lam[kMaxL];               // lambda of every drafter row
   int nc[2];                      // candidates of a level (phase 2, double-buffered)
   unsigned long long tau;         // the smallest key of a full A (phase 2)
 };
@@ -160,19 +163,22 @@ constexpr int kCluster = 8;
 // set C of a level are double-buffered.  Per entry: key, the index of its own children's
 // context (kNoCtx at depth L), its candidate index j, and its parent's node index.
 struct P2Layout {
-  size_t akey, axc, apid, aj, ckey, cxc, cpid, cj, rk, bytes;
-  __host__ __device__ P2Layout(int N, int bf) {
-    const size_t na = N, nc = static_cast<size_t>(N) * bf;
+  size_t akey, axc, apid, aj, ckey, cxc, cpid, cj, rk, rkc, bytes;
+  int nc;  // capacity of one candidate buffer: every child of max(N, W) parents
+  __host__ __device__ P2Layout(int N, int bf, int W) {
+    const size_t na = N;
+    nc = (N > W ? N : W) * bf;
     size_t o = 0;
     akey = o;  o += 2 * na * 8;
-    ckey = o;  o += 2 * nc * 8;
+    ckey = o;  o += 2 * static_cast<size_t>(nc) * 8;
     axc = o;   o += 2 * na * 4;
-    cxc = o;   o += 2 * nc * 4;
+    cxc = o;   o += 2 * static_cast<size_t>(nc) * 4;
     apid = o;  o += align_up(2 * na * 2, 4);
-    cpid = o;  o += align_up(2 * nc * 2, 4);
+    cpid = o;  o += align_up(2 * static_cast<size_t>(nc) * 2, 4);
     rk = o;    o += align_up((na + nc) * 2, 4);
+    rkc = o;   o += align_up(static_cast<size_t>(nc) * 2, 4);
     aj = o;    o += align_up(2 * na, 4);
-    cj = o;    o += align_up(2 * nc, 4);
+    cj = o;    o += align_up(2 * static_cast<size_t>(nc), 4);
     bytes = align_up(o, 16);
   }
 };
@@ -193,13 +199,14 @@ constexpr uint32_t kNoCtx = 0xFFFFFFFFu;
 // Returns the node count (root included).
 __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigned char* p2,
                              int tid) {
-  const int L = a.L, k = a.k, N = a.N, nb = a.bf;
+  const int L = a.L, k = a.k, N = a.N, nb = a.bf, W = a.W;
+  const bool beam = a.policy == PRESTO_SEARCH_BEAM;
   const int cs = a.use_table ? k * k : 1;
   const int cap = N - 1;  // non-root nodes
   const int lane = tid & 31;
-  const P2Layout ly(N, nb);
-  const int NC = N * nb;
-  // buffer u of each A field starts at u * N, of each C field at u * N * nb
+  const P2Layout ly(N, nb, W);
+  const int NC = ly.nc;
+  // buffer u of each A field starts at u * N, of each C field at u * NC
   uint64_t* const akey = reinterpret_cast<uint64_t*>(p2 + ly.akey);
   uint32_t* const axc = reinterpret_cast<uint32_t*>(p2 + ly.axc);
   int16_t* const apid = reinterpret_cast<int16_t*>(p2 + ly.apid);
@@ -209,17 +216,26 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
   int16_t* const cpid = reinterpret_cast<int16_t*>(p2 + ly.cpid);
   uint8_t* const cj = p2 + ly.cj;
   int16_t* const rk = reinterpret_cast<int16_t*>(p2 + ly.rk);
+  int16_t* const rkc = reinterpret_cast<int16_t*>(p2 + ly.rkc);
 
-  // Child c of a node with score Sp, children context x, candidate index pj and
-  // node index pnode, at depth dc: its key, context and candidate index.
-  auto child = [&](uint32_t x, float Sp, int pj, int pnode, int dc, int c, uint64_t& key,
+  // Child c of a node with score Sp, children context x and candidate index pj, at
+  // depth dc; `pfield` fills the key's last field (255 - the parent's position among
+  // the parents of its level).  Returns the key, context and candidate index.
+  auto child = [&](uint32_t x, float Sp, int pj, int pfield, int dc, int c, uint64_t& key,
                    uint32_t& xc, int& jc) {
     const uint2 kd = kids[x * nb + c];
     key = (static_cast<uint64_t>(ordered(__fadd_rn(Sp, __uint_as_float(kd.x)))) << 32) |
-          (kd.y & ~0xFFu) | static_cast<uint32_t>(255 - pnode);
+          (kd.y & ~0xFFu) | static_cast<uint32_t>(255 - pfield);
     jc = static_cast<int>(kd.y & 0xFFu);
     xc = dc >= L ? kNoCtx
                  : static_cast<uint32_t>(dc * cs + (!a.use_table ? 0 : (dc == 1 ? jc : pj * k + jc)));
+  };
+  // Reserve `keep`-many candidate slots of buffer u, one atomic per warp (all lanes).
+  auto reserve = [&](bool keep, int u) {
+    const unsigned bal = __ballot_sync(0xffffffffu, keep);
+    int base = 0;
+    if (lane == 0 && bal) base = atomicAdd(&sm.nc[u], __popc(bal));
+    return __shfl_sync(0xffffffffu, base, 0) + __popc(bal & ((1u << lane) - 1u));
   };
 
   // level 1: the root's children (A is empty, so every one is a candidate)
@@ -236,9 +252,11 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
   if (tid == 0) sm.nc[1] = 0;
   __syncthreads();
   int na = 0, m = cap > 0 ? nb : 0, cur = 0, cc = 0;
-  uint64_t tau = 0ull;  // candidates need key > tau (0: A not yet full)
+  int tsize = 1 + m;    // |T|, root included (beam search stops once it reaches N)
+  uint64_t tau = 0ull;  // the smallest key of A once A is full (0: not yet full)
   for (int step = 0; m > 0; ++step) {
-    // ---- ranks in A u C by (key desc, position asc); A is sorted
+    // ---- ranks in A u C by (key desc, position asc); A is sorted.  rkc: the rank of
+    // a candidate among the candidates alone (beam search keeps the W best)
     const uint64_t* C = ckey + cc * NC;
     const int ne = na + m;
     for (int e = tid; e < ne; e += kThreads) {
@@ -256,11 +274,13 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
           if (akey[cur * N + mid] >= ke) lo = mid + 1;
           else hi = mid;
         }
-        r = lo;
+        int rc = 0;
         for (int i = 0; i < m; ++i) {
           const uint64_t ki = C[i];
-          r += ki > ke || (ki == ke && i < ci);
+          rc += ki > ke || (ki == ke && i < ci);
         }
+        rkc[ci] = static_cast<int16_t>(rc);
+        r = lo + rc;
       }
       rk[e] = static_cast<int16_t>(r < cap ? r : cap);
       if (r == cap - 1) sm.tau = e < na ? akey[cur * N + e] : C[e - na];  // the new A's last key
@@ -269,8 +289,9 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
     __syncthreads();
     if (ne >= cap) tau = sm.tau;  // the new A is full: its smallest key
     // ---- the cap largest become the new A (parent indices follow their ranks), and
-    // the new nodes, the survivors of C, generate the next level's candidates: their
-    // children with key > tau, the smallest key of the new A once it is full
+    // the next level's candidates are generated:
+    //   best-first: children of the new nodes that entered A, with key > tau;
+    //   beam: children of the W best candidates (the beam), all of them, while |T| < N
     const int nxt = cur ^ 1, cn = cc ^ 1;
     for (int e = tid; e < ne; e += kThreads) {
       const int r = rk[e];
@@ -291,36 +312,38 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
         const int pr = rk[pid - 1];
         if (pr >= cap || pr >= r) report(a.dev_status, PRESTO_DEV_BAD_PARENT);  // s > 0 input
         pid = pr < cap ? pr + 1 : 0;
+      } else if (pid < 0) {  // a parent outside A: cannot happen when every s <= 0
+        report(a.dev_status, PRESTO_DEV_BAD_PARENT);
+        pid = 0;
       }
       apid[nxt * N + r] = static_cast<int16_t>(pid);
     }
-    // (candidate, child) pairs over the whole CTA; slots reserved per warp
-    const int pairs = m * nb;
+    const bool grow = !beam || tsize < N;  // warp-uniform
+    const int pairs = grow ? m * nb : 0;
     const int iters = (pairs + kThreads - 1) / kThreads;  // uniform, for the warp scans
     for (int it = 0; it < iters; ++it) {
       const int q = it * kThreads + tid;
       const int ci = q / nb, c = q - ci * nb;
       const int r = q < pairs ? rk[na + ci] : cap;
-      const uint32_t xe = r < cap ? cxc[cc * NC + ci] : kNoCtx;
+      const int rc = q < pairs ? rkc[ci] : W;
+      const bool parent = beam ? rc < W : r < cap;
+      const uint32_t xe = parent ? cxc[cc * NC + ci] : kNoCtx;
       uint64_t key = 0ull;
       uint32_t xc = kNoCtx;
       int jc = 0;
-      if (xe != kNoCtx) {  // a new node below depth L
+      if (xe != kNoCtx) {  // a parent below depth L
         const uint64_t ke = C[ci];
         const int dc = 64 - static_cast<int>((ke >> 26) & 63u);  // the children's depth
-        child(xe, unordered(static_cast<uint32_t>(ke >> 32)), cj[cc * NC + ci], r + 1, dc, c,
-              key, xc, jc);
+        child(xe, unordered(static_cast<uint32_t>(ke >> 32)), cj[cc * NC + ci],
+              beam ? rc : r + 1, dc, c, key, xc, jc);
       }
-      const bool keep = key > tau;
-      const unsigned bal = __ballot_sync(0xffffffffu, keep);
-      int base = 0;
-      if (lane == 0 && bal) base = atomicAdd(&sm.nc[cn], __popc(bal));
-      base = __shfl_sync(0xffffffffu, base, 0) + __popc(bal & ((1u << lane) - 1u));
+      const bool keep = key != 0ull && (beam || key > tau);
+      const int slot = reserve(keep, cn);
       if (keep) {
-        ckey[cn * NC + base] = key;
-        cxc[cn * NC + base] = xc;
-        cpid[cn * NC + base] = static_cast<int16_t>(r + 1);
-        cj[cn * NC + base] = static_cast<uint8_t>(jc);
+        ckey[cn * NC + slot] = key;
+        cxc[cn * NC + slot] = xc;
+        cpid[cn * NC + slot] = static_cast<int16_t>(r < cap ? r + 1 : -1);
+        cj[cn * NC + slot] = static_cast<uint8_t>(jc);
       }
     }
     na = ne < cap ? ne : cap;
@@ -328,21 +351,117 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
     cc = cn;
     __syncthreads();
     m = sm.nc[cc];
+    tsize += m;
   }
-  // ---- write the tree: node 0 is the root, node r + 1 is A[r]
+
+  // ---- Alg. 2 as printed: the nodes are expanded in the lazy order above (node 0
+  // the root, node r + 1 = A[r]) until |T| = 1 + (their children) reaches N; the
+  // output is those X nodes, then the best of their children not expanded
+  int head = na + 1, ntail = 0;  // rows from A (root included), rows from the tail
+  if (a.policy == PRESTO_SEARCH_EAGER) {
+    __syncthreads();  // every thread has read the loop's last counter
+    if (tid == 0) {
+      int cnt = 1, x = 0;
+      while (cnt < N && x <= na) {
+        const int d = x == 0 ? 0 : 63 - static_cast<int>((akey[cur * N + x - 1] >> 26) & 63u);
+        cnt += d < L ? nb : 0;
+        ++x;
+      }
+      sm.nc[0] = x;
+      sm.nc[1] = 0;
+    }
+    __syncthreads();
+    const int X = sm.nc[0];
+    // X = 0 (N = 1): nothing expanded, the root alone; X > na: the whole tree
+    if (X >= 1 && X <= na) {
+      head = X;
+      // the children of nodes 0 .. X-1 that are not among nodes 1 .. X-1
+      const int pairs = X * nb;
+      const int iters = (pairs + kThreads - 1) / kThreads;
+      uint64_t* const F = ckey + cc * NC;  // the last level's buffer is free now
+      for (int it = 0; it < iters; ++it) {
+        const int q = it * kThreads + tid;
+        const int i = q / nb, c = q - i * nb;
+        uint64_t key = 0ull;
+        uint32_t xc = kNoCtx;
+        int jc = 0;
+        if (q < pairs) {
+          uint64_t ke = 0ull;
+          uint32_t x = 0u;
+          int pj = 0, d = 0;
+          if (i > 0) {
+            ke = akey[cur * N + i - 1];
+            x = axc[cur * N + i - 1];
+            pj = aj[cur * N + i - 1];
+            d = 63 - static_cast<int>((ke >> 26) & 63u);
+          }
+          if (d < L) {
+            child(x, i == 0 ? 0.f : unordered(static_cast<uint32_t>(ke >> 32)), pj, i, d + 1, c,
+                  key, xc, jc);
+            // expanded already: one of A[0 .. X-2], the same (S, depth, token) under the
+            // same parent (A's last key field dates from its own level, so compare
+            // the node's parent instead)
+            int lo = 0, hi = X - 1;
+            while (lo < hi) {
+              const int mid = (lo + hi) >> 1;
+              if ((akey[cur * N + mid] >> 8) > (key >> 8)) lo = mid + 1;
+              else hi = mid;
+            }
+            for (; lo < X - 1 && (akey[cur * N + lo] >> 8) == (key >> 8); ++lo)
+              if (apid[cur * N + lo] == i) key = 0ull;
+          }
+        }
+        const bool keep = key != 0ull;
+        const int slot = reserve(keep, 1);
+        if (keep) {
+          F[slot] = key;
+          cpid[cc * NC + slot] = static_cast<int16_t>(i);
+        }
+      }
+      __syncthreads();
+      const int nf = sm.nc[1];
+      ntail = nf < N - X ? nf : N - X;
+      for (int e = tid; e < nf; e += kThreads) {
+        const uint64_t ke = F[e];
+        int r = 0;
+        for (int i2 = 0; i2 < nf; ++i2) r += F[i2] > ke || (F[i2] == ke && i2 < e);
+        rk[e] = static_cast<int16_t>(r);
+      }
+      __syncthreads();
+      // the tail rows, in rank order, into A's buffer beyond the head
+      for (int e = tid; e < nf; e += kThreads) {
+        const int r = rk[e];
+        if (r >= ntail) continue;
+        akey[(cur ^ 1) * N + r] = F[e];
+        apid[(cur ^ 1) * N + r] = cpid[cc * NC + e];
+      }
+      __syncthreads();
+    }
+  }
+
+  // ---- write the tree: node 0 is the root, node r + 1 is A[r] for r + 1 < head, then
+  // the tail rows
   for (int i = tid; i < N; i += kThreads) {
     const size_t o = static_cast<size_t>(blockIdx.x / kCluster) * N + i;
+    uint64_t ke = 0ull;
+    int pid = -1;
+    if (i > 0 && i < head) {
+      ke = akey[cur * N + i - 1];
+      pid = apid[cur * N + i - 1];
+    } else if (i >= head && i < head + ntail) {
+      ke = akey[(cur ^ 1) * N + i - head];
+      pid = apid[(cur ^ 1) * N + i - head];
+    }
     if (i == 0) {
       a.node_token[o] = sm.ctx1;
       a.node_parent[o] = -1;
       a.node_depth[o] = 0;
       a.node_score[o] = 0.f;
-    } else if (i <= na) {
-      const uint64_t ke = akey[cur * N + i - 1];
+    } else if (ke != 0ull) {
       const uint32_t lo = static_cast<uint32_t>(ke);
       a.node_token[o] = 0x3FFFF - static_cast<int>((lo >> 8) & 0x3FFFFu);
       a.node_depth[o] = 63 - static_cast<int>((lo >> 26) & 63u);
-      a.node_parent[o] = apid[cur * N + i - 1];
+      a.node_parent[o] = pid;
       a.node_score[o] = unordered(static_cast<uint32_t>(ke >> 32));
     } else {
       a.node_token[o] = -1;
@@ -351,7 +470,7 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
       a.node_score[o] = -INFINITY;
     }
   }
-  return na + 1;
+  return head + ntail;
 }
 
 __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
@@ -388,6 +507,14 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
     sm.cid[d][j] = t;
     sm.clq[d][j] = a.logq[(static_cast<size_t>(b) * L + d) * k + j];
   }
+  for (int d = tid; d < L; d += kThreads) {
+    float lam = a.lambda_d ? a.lambda_d[static_cast<size_t>(b) * L + d] : a.lambda;
+    if (!(lam >= 0.f)) {  // negative or NaN: scores could turn positive
+      if (rank == 0) report(a.dev_status, PRESTO_DEV_POSITIVE_SCORE);
+      lam = 0.f;
+    }
+    sm.lam[d] = lam;
+  }
   if (tid == 0) {
     sm.ctx0 = a.ctx2[2 * b];
     sm.ctx1 = a.ctx2[2 * b + 1];
@@ -413,18 +540,20 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   for (int f0 = tid; f0 < my; f0 += kThreads * kBatch) {
     uint64_t key[kBatch];
     uint32_t h[kBatch];
-    float lq[kBatch];
+    float lq[kBatch], lam[kBatch];
 #pragma unroll
     for (int q = 0; q < kBatch; ++q) {
       const int f = f0 + q * kThreads;
       key[q] = PRESTO_NGRAM3_EMPTY;
       h[q] = 0;
       lq[q] = 0.f;
+      lam[q] = 0.f;
       if (f >= my) continue;
       const int gl = f / k, j = f - gl * k;
       int d, ci;
       decode_ctx(g0 + gl, k, use_table, d, ci);
       lq[q] = sm.clq[d][j];
+      lam[q] = sm.lam[d];
       if (!use_table) continue;
       int ta, tb;
       if (d == 0) {
@@ -489,7 +618,7 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
         if (!done)  // a chain longer than the window: continue slot by slot
           lr = probe_from(a.keys, a.logrho, a.cap_mask, a.miss, key[q],
                           (h[q] + 1 + kWin) & a.cap_mask);
-        sc = __fadd_rn(__fmul_rn(a.lambda, lr), lq[q]);
+        sc = __fadd_rn(__fmul_rn(lam[q], lr), lq[q]);
       }
       if (sc > 0.f) report(a.dev_status, PRESTO_DEV_POSITIVE_SCORE);
       if (nb == k) {  // every candidate is kept
@@ -564,9 +693,9 @@ extern "C" int presto_ngram3_insert(const presto_ngram3* t, const uint64_t* keys
 
 namespace {
 // phase-1 staging area of each CTA, reused by the leader for phase 2
-size_t stage_bytes(int per_cta, int k, int N, int bf) {
+size_t stage_bytes(int per_cta, int k, int N, int bf, int W) {
   const size_t st = align_up(static_cast<size_t>(per_cta) * k * 4, 16);
-  const size_t p2 = P2Layout(N, bf).bytes;
+  const size_t p2 = P2Layout(N, bf, W).bytes;
   return st > p2 ? st : p2;
 }
 int contexts_all(int L, int k, int use_table) {
@@ -575,14 +704,18 @@ int contexts_all(int L, int k, int use_table) {
 }
 }  // namespace
 
-extern "C" size_t presto_build_workspace(int B, int L, int k, int N) {
-  if (B < 1 || L < 1 || k < 1 || N < 1) return 0;
+extern "C" size_t presto_build_workspace_ex(int B, int L, int k, int N, int beam_width) {
+  if (B < 1 || L < 1 || k < 1 || N < 1 || beam_width < 1) return 0;
   // The leader CTA keeps the tables in shared memory when they fit; otherwise they
   // live here (sized for the prefix-signal case, the larger one).
   const TableLayout tl(L, k, k, 1);
   const int per = (contexts_all(L, k, 1) + kCluster - 1) / kCluster;
-  const size_t smem = tl.bytes + stage_bytes(per, k, N, k);
+  const size_t smem = tl.bytes + stage_bytes(per, k, N, k, beam_width);
   return smem <= kDynSmemBudget ? 256 : align_up(B * tl.bytes, 256);
+}
+
+extern "C" size_t presto_build_workspace(int B, int L, int k, int N) {
+  return presto_build_workspace_ex(B, L, k, N, 1);
 }
 
 extern "C" int presto_score_build_tree(const int32_t* topk_ids, const float* topk_logq, int B,
@@ -592,11 +725,28 @@ extern "C" int presto_score_build_tree(const int32_t* topk_ids, const float* top
                                        int32_t* node_depth, float* node_score,
                                        int32_t* n_nodes, void* ws, size_t ws_bytes,
                                        int32_t* dev_status, presto_stream_t stream) {
+  return presto_score_build_tree_ex(topk_ids, topk_logq, B, L, k, b, ctx2, ngram, lambda,
+                                    nullptr, PRESTO_SEARCH_BEST_FIRST, 1, N, node_token,
+                                    node_parent, node_depth, node_score, n_nodes, ws, ws_bytes,
+                                    dev_status, stream);
+}
+
+extern "C" int presto_score_build_tree_ex(const int32_t* topk_ids, const float* topk_logq,
+                                          int B, int L, int k, int b, const int32_t* ctx2,
+                                          const presto_ngram3* ngram, float lambda,
+                                          const float* lambda_d, int policy, int beam_width,
+                                          int N, int32_t* node_token, int32_t* node_parent,
+                                          int32_t* node_depth, float* node_score,
+                                          int32_t* n_nodes, void* ws, size_t ws_bytes,
+                                          int32_t* dev_status, presto_stream_t stream) {
   PRESTO_CHECK_ARG(topk_ids && topk_logq && ctx2 && node_token && node_parent && node_depth &&
                    node_score && n_nodes);
   PRESTO_CHECK_ARG(B >= 1 && L >= 1 && k >= 1 && b >= 1 && N >= 1 && b <= k);
   PRESTO_CHECK_ARG(lambda >= 0.f && lambda == lambda);
-  PRESTO_CHECK_LIMIT(L <= kMaxL && k <= kMaxK && N <= kMaxN);
+  PRESTO_CHECK_ARG(policy == PRESTO_SEARCH_BEST_FIRST || policy == PRESTO_SEARCH_BEAM ||
+                   policy == PRESTO_SEARCH_EAGER);
+  PRESTO_CHECK_ARG(beam_width >= 1);
+  PRESTO_CHECK_LIMIT(L <= kMaxL && k <= kMaxK && N <= kMaxN && beam_width <= kMaxN);
   if (ngram) {
     PRESTO_CHECK_ARG(ngram->keys && ngram->logrho);
     PRESTO_CHECK_ARG(ngram->log2_cap >= 4 && ngram->log2_cap <= 30);
@@ -614,6 +764,9 @@ extern "C" int presto_score_build_tree(const int32_t* topk_ids, const float* top
     a.miss = ngram->miss_logrho;
   }
   a.lambda = lambda;
+  a.lambda_d = lambda_d;
+  a.policy = policy;
+  a.W = beam_width;
   a.L = L;
   a.k = k;
   a.bf = b;
@@ -621,7 +774,7 @@ extern "C" int presto_score_build_tree(const int32_t* topk_ids, const float* top
   a.nctx_all = contexts_all(L, k, a.use_table);
   a.per_cta = (a.nctx_all + kCluster - 1) / kCluster;
   const TableLayout tl(L, k, b, a.use_table);
-  const size_t sb = stage_bytes(a.per_cta, k, N, b);
+  const size_t sb = stage_bytes(a.per_cta, k, N, b, beam_width);
   a.tables_in_smem = tl.bytes + sb <= kDynSmemBudget;
   if (!a.tables_in_smem) {
     if (!ws || reinterpret_cast<uintptr_t>(ws) % 16 || ws_bytes < static_cast<size_t>(B) * tl.bytes)

@@ -168,3 +168,33 @@ def test_eager_is_the_lazy_prefix_then_its_best_unexpanded_children():
                     _check(got, _as_rows(chosen, by_path, int(ctx[0, 1])), len(chosen))
                     cases += 1
     assert cases >= 40
+
+
+def test_per_row_lambda_matches_enumeration_and_special_cases():
+    """App. F: a lambda_d per position.  Best-first, beam and eager with a [B, L]
+    lambda against exhaustive enumeration scored from scratch; a constant array
+    equals the scalar; a zero row is prefix-blind at that depth."""
+    rng = np.random.default_rng(11)
+    for trial in range(30):
+        L, k = 4, 3
+        ids, logq, ctx, table = _random_case(rng, L, k, 6, True)
+        lam_d = rng.choice([0.0, 0.125, 0.25, 0.5, 1.0], size=(1, L))
+        N = int(rng.integers(2, 20))
+        want = O.brute_force_tree(ids, logq, ctx, table, -2.0, lam_d, k, N, "fp32")
+        got = O.best_first_tree(ids, logq, ctx, table, -2.0, lam_d, k, N, "fp32")
+        for key in KEYS:
+            np.testing.assert_array_equal(got[key], want[key], err_msg=key)
+        const = np.full((1, L), 0.25)
+        for fn, extra in ((O.best_first_tree, ()), (O.eager_tree, ()),
+                          (O.beam_search_tree, (3,))):
+            a = fn(ids, logq, ctx, table, -2.0, const, k, N, *extra)
+            s = fn(ids, logq, ctx, table, -2.0, 0.25, k, N, *extra)
+            for key in KEYS + ("score",):
+                np.testing.assert_array_equal(a[key], s[key], err_msg=key)
+    # a zero row: depth-1 scores are log q alone
+    ids, logq, ctx, table = _random_case(rng, 3, 3, 6, True)
+    lam_d = np.array([[0.0, 0.5, 0.5]])
+    t = O.best_first_tree(ids, logq, ctx, table, -2.0, lam_d, 3, 4, "fp64")
+    for i in range(1, int(t["n_nodes"][0])):
+        if t["depth"][0, i] == 1:
+            assert t["score"][0, i] == logq[0, 0, t["rank"][0, i]]

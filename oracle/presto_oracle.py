@@ -77,6 +77,34 @@ def topk_logsoftmax(logits, k: int):
     return ids, logq, lse
 
 
+def drafter_entropy(logits):
+    """H_d = -sum_w q_d(w) log q_d(w) of each row (App. F), q_d the softmax of the
+    row (§2.3 marginal).  Entries of -inf have q = 0 and add nothing (0 log 0 = 0).
+
+    logits: array [R, V] of finite values or -inf, each row with a finite entry.
+    Returns float64 [R] in nats.
+    """
+    x = np.asarray(logits, dtype=np.float64)
+    m = x.max(axis=1, keepdims=True)
+    z = x - m
+    e = np.exp(z)
+    Z = e.sum(axis=1)
+    logq = z - np.log(Z)[:, None]
+    q = e / Z[:, None]
+    with np.errstate(invalid="ignore"):
+        terms = np.where(q > 0.0, q * logq, 0.0)
+    return -terms.sum(axis=1)
+
+
+def entropy_adaptive_lambda(H, beta: float, C: float):
+    """lambda_d(H_d) = beta * H_d / (H_d + C) (App. F; beta > 0 the largest
+    correction strength, C > 0 the stabilising constant).  float64."""
+    if not (beta > 0 and C > 0):
+        raise ValueError("need beta > 0 and C > 0")
+    H = np.asarray(H, dtype=np.float64)
+    return beta * H / (H + C)
+
+
 # ---------------------------------------------------------------------------
 # Step 2: prefix-aligned token score (§4.1, Eq. prefix-aligned-conditional and
 # Eq. path-score): s_{d,t}(c_d) = log q_d(t) + lambda_d log rho_d(t | c_d).

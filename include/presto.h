@@ -5,6 +5,7 @@
  * scoring and priority-based tree search):
  *
  *   presto_topk             per-position log-softmax and top-k of the drafter logits
+ *   presto_topk_entropy     the same, plus each row's entropy and adaptive lambda_d
  *   presto_score_build_tree prefix-aligned scores + best-first tree up to N nodes
  *                           (_ex: beam search / printed Alg. 2, per-position lambda)
  *   presto_tree_mask        ancestor bitmask and position ids of the tree tokens
@@ -122,6 +123,28 @@ int presto_topk(const void* logits, int dtype, int B, int L, int V, long long ro
 int presto_topk_noalloc(const void* logits, int dtype, int B, int L, int V,
                         long long row_stride, int k, int32_t* topk_ids, float* topk_logq,
                         float* lse, int32_t* dev_status, presto_stream_t stream);
+
+/*
+ * presto_topk_entropy - presto_topk that also yields each row's entropy and the
+ * entropy-adaptive lambda_d of App. F, in the same single pass over the logits.
+ *
+ *   H_d = -sum_w q_d(w) log q_d(w)  (nats; q_d the row's softmax, §2.3)
+ *   lambda_d(H_d) = beta * H_d / (H_d + C)
+ *
+ *   beta, C     > 0 and finite when lambda_d is given (the largest correction
+ *               strength and the stabilising constant; the paper fixes neither).
+ *   entropy     [B, L] float32 out, nullable: H_d of every row.
+ *   lambda_d    [B, L] float32 out, nullable: lambda_d(H_d), float32 with correctly
+ *               rounded multiply, add and divide; it is the layout that
+ *               presto_score_build_tree_ex takes as its lambda_d.
+ * At least one of entropy, lambda_d is non-null.  Every other argument and result
+ * is as presto_topk.  Where presto_topk reports PRESTO_DEV_NONFINITE for a row,
+ * its entropy and lambda_d are unspecified.
+ */
+int presto_topk_entropy(const void* logits, int dtype, int B, int L, int V,
+                        long long row_stride, int k, float beta, float C, int32_t* topk_ids,
+                        float* topk_logq, float* lse, float* entropy, float* lambda_d, void* ws,
+                        size_t ws_bytes, int32_t* dev_status, presto_stream_t stream);
 
 /*
  * Trigram prefix signal rho_d(t | t_{d-2}, t_{d-1}) (§4.1; the paper instantiates

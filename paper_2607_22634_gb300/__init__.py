@@ -22,6 +22,8 @@ from ._lib import (  # noqa: F401
     presto_build_workspace,
     presto_score_build_tree,
     presto_topk,
+    presto_topk_entropy,
+    presto_topk_noalloc,
     presto_topk_workspace,
     presto_tree_attention,
     presto_tree_mask,

@@ -48,6 +48,8 @@ _SIGS = {
     "presto_topk": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, _P, _P, _P, _P,
                          ctypes.c_size_t, _P, _P]),
     "presto_topk_noalloc": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, _P, _P, _P, _P, _P]),
+    "presto_topk_entropy": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, ctypes.c_float,
+                                 ctypes.c_float, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "presto_ngram3_clear": (_I, [ctypes.POINTER(Ngram3), _P]),
     "presto_ngram3_insert": (_I, [ctypes.POINTER(Ngram3), _P, _P, _I, _P, _P]),
     "presto_build_workspace": (ctypes.c_size_t, [_I, _I, _I, _I]),
@@ -172,6 +174,44 @@ def presto_topk_noalloc(logits, k, topk_ids, topk_logq, lse=None, dev_status=Non
                                     _stream(stream))
     _check(st, "presto_topk_noalloc")
     return topk_ids, topk_logq, lse
+
+
+def presto_topk_entropy(logits, k, beta=None, C=None, topk_ids=None, topk_logq=None, lse=None,
+                        entropy=None, lambda_d=None, ws=None, dev_status=None, stream=None,
+                        with_lse=True, with_entropy=True, with_lambda=True):
+    """presto_topk plus each row's entropy H_d and lambda_d = beta H_d / (H_d + C)
+    (App. F).  Returns (topk_ids, topk_logq, lse, entropy, lambda_d); lambda_d is
+    None unless beta and C are given."""
+    if logits.dim() != 3 or logits.stride(2) != 1 or logits.stride(0) != logits.shape[1] * logits.stride(1):
+        raise ValueError("logits must be [B, L, V] with unit last stride and packed rows")
+    B, L, V = logits.shape
+    dtype = {torch.float32: PRESTO_F32, torch.bfloat16: PRESTO_BF16}.get(logits.dtype)
+    if dtype is None:
+        raise ValueError("logits must be float32 or bfloat16")
+    dev = logits.device
+    f32 = torch.float32
+    topk_ids = torch.empty(B, L, k, dtype=torch.int32, device=dev) if topk_ids is None else topk_ids
+    topk_logq = torch.empty(B, L, k, dtype=f32, device=dev) if topk_logq is None else topk_logq
+    if lse is None and with_lse:
+        lse = torch.empty(B, L, dtype=f32, device=dev)
+    if entropy is None and with_entropy:
+        entropy = torch.empty(B, L, dtype=f32, device=dev)
+    adaptive = beta is not None and C is not None
+    if lambda_d is None and with_lambda and adaptive:
+        lambda_d = torch.empty(B, L, dtype=f32, device=dev)
+    _need(topk_ids, torch.int32, (B, L, k), "topk_ids")
+    _need(topk_logq, f32, (B, L, k), "topk_logq")
+    for t, name in ((lse, "lse"), (entropy, "entropy"), (lambda_d, "lambda_d")):
+        if t is not None:
+            _need(t, f32, (B, L), name)
+    ws, nws = _ws(presto_topk_workspace(B, L, V, k), dev, ws)
+    st = load().presto_topk_entropy(_ptr(logits), dtype, B, L, V, logits.stride(1), k,
+                                    float(beta) if adaptive else 0.0,
+                                    float(C) if adaptive else 0.0, _ptr(topk_ids), _ptr(topk_logq),
+                                    _ptr(lse), _ptr(entropy), _ptr(lambda_d), _ptr(ws), nws,
+                                    _ptr(dev_status), _stream(stream))
+    _check(st, "presto_topk_entropy")
+    return topk_ids, topk_logq, lse, entropy, lambda_d
 
 
 # ------------------------------------------------------------------ trigram table

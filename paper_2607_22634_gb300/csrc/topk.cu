@@ -19,6 +19,10 @@
 //         survivors fit.
 //   * The leader CTA of the cluster merges the spans' (max, Σexp) pairs and top-k
 //     lists and writes the row.
+//   * With ENT the same pass also yields the row's entropy (App. F): next to
+//     s = Σ 2^u, u = x log2e - max2, each thread sums t = Σ 2^u u, and the merges
+//     carry t along (when the reference maximum drops by δ, t -> 2^δ (t + δ s)).
+//     Then H = ln s - ln2 t / s, and lambda_d = beta H / (H + C).
 #include <cuda_bf16.h>
 
 #include <cooperative_groups.h>
@@ -110,6 +114,28 @@ __device__ __forceinline__ void merge_ms(float& m2, float& s, float n2, float t)
   s = s * ex2(m2 - M) + t * ex2(n2 - M);
   m2 = M;
 }
+// The same with the entropy sums t = Σ 2^u u, u = x log2e - max: moving a pair's
+// reference maximum from m to M scales s by 2^(m-M) and t to 2^(m-M) (t + (m-M) s).
+// A pair with maximum -inf holds nothing (s = t = 0) and is skipped.
+__device__ __forceinline__ void merge_mst(float& m2, float& s, float& t, float n2, float s2,
+                                          float t2) {
+  const float M = fmaxf(m2, n2);
+  if (M == -INFINITY) return;
+  float so = 0.f, to = 0.f;
+  if (m2 != -INFINITY) {
+    const float f = ex2(m2 - M);
+    so = s * f;
+    to = f * fmaf(m2 - M, s, t);
+  }
+  if (n2 != -INFINITY) {
+    const float f = ex2(n2 - M);
+    so = fmaf(s2, f, so);
+    to = fmaf(f, fmaf(n2 - M, s2, t2), to);
+  }
+  s = so;
+  t = to;
+  m2 = M;
+}
 
 struct Plan {
   int rows, parts, vpt, vmax;  // vpt: vectors per thread; vmax: the kernel's register bound
@@ -123,6 +149,9 @@ struct Args {
   int32_t* topk_ids;
   float* topk_logq;
   float* lse;
+  float* entropy;   // ENT: [rows] H in nats, nullable
+  float* lambda_d;  // ENT: [rows] beta H / (H + C), nullable
+  float beta, C;
   int32_t* dev_status;
 };
 
@@ -132,6 +161,8 @@ struct Smem {
   unsigned long long part[kMaxParts][kMaxK];    // leader: the cluster's lists
   float2 part_ms[kMaxParts];                    // leader: the cluster's (max, sum)
   float2 warp_ms[kWarps];                       // (max log2, sum) per warp
+  float warp_t[kWarps];                         // ENT: entropy sum per warp
+  float part_t[kMaxParts];                      // ENT leader: the cluster's entropy sums
   float warp_max[kWarps];                       // plain maxima, for tau
   unsigned long long thr;                       // key threshold of the current round
   int count;
@@ -150,7 +181,7 @@ __device__ __forceinline__ void rank_keys(const unsigned long long* e, int M, in
   }
 }
 
-template <typename T, int VMAX>
+template <typename T, int VMAX, bool ENT>
 __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const Args a) {
   namespace cg = cooperative_groups;
   using E = Elem<T>;
@@ -195,27 +226,58 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
 #pragma unroll
   for (int i = 0; i < VMAX; ++i) mt = fmaxf(mt, E::vmax(d[i]));
   const float m2 = mt * kLog2e;
-  float st = 0.f;
+  float st = 0.f, tt = 0.f;  // tt (ENT): Σ 2^u u
   if (mt != -INFINITY) {
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    if constexpr (!ENT) {
 #pragma unroll
-    for (int i = 0; i < VMAX; ++i) {
+      for (int i = 0; i < VMAX; ++i) {
 #pragma unroll
-      for (int e = 0; e < n; ++e) acc[e & 3] += ex2(fmaf(E::value(d[i], e), kLog2e, -m2));
+        for (int e = 0; e < n; ++e) acc[e & 3] += ex2(fmaf(E::value(d[i], e), kLog2e, -m2));
+      }
+      st = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      if (xid >= 0) st += ex2(fmaf(xval, kLog2e, -m2));
+    } else {
+      // u is clamped at -256: 2^u flushes to 0 there, so -inf entries add 0 to both
+      float tac[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int i = 0; i < VMAX; ++i) {
+#pragma unroll
+        for (int e = 0; e < n; ++e) {
+          const float u = fmaxf(fmaf(E::value(d[i], e), kLog2e, -m2), -256.f);
+          const float p = ex2(u);
+          acc[e & 3] += p;
+          tac[e & 3] = fmaf(p, u, tac[e & 3]);
+        }
+      }
+      st = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      tt = (tac[0] + tac[1]) + (tac[2] + tac[3]);
+      if (xid >= 0) {
+        const float u = fmaxf(fmaf(xval, kLog2e, -m2), -256.f);
+        const float p = ex2(u);
+        st += p;
+        tt = fmaf(p, u, tt);
+      }
     }
-    st = (acc[0] + acc[1]) + (acc[2] + acc[3]);
-    if (xid >= 0) st += ex2(fmaf(xval, kLog2e, -m2));
   }
   // ---- warp: (max, sum) and the plain maximum
   const uint32_t wm_o = __reduce_max_sync(kFull, ordered(mt));
   const float wm = unordered(wm_o);
   const float wm2 = wm * kLog2e;
-  float ws = (mt == -INFINITY) ? 0.f : st * ex2(m2 - wm2);
+  const float fw = (mt == -INFINITY) ? 0.f : ex2(m2 - wm2);
+  float ws = st * fw;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) ws += __shfl_xor_sync(kFull, ws, off);
+  float wt = 0.f;
+  if constexpr (ENT) {
+    wt = (mt == -INFINITY) ? 0.f : fw * fmaf(m2 - wm2, st, tt);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) wt += __shfl_xor_sync(kFull, wt, off);
+  }
   if (lane == 0) {
     sh.warp_ms[warp] = make_float2(wm == -INFINITY ? -INFINITY : wm2, ws);
     sh.warp_max[warp] = wm;
+    if constexpr (ENT) sh.warp_t[warp] = wt;
   }
   if (tid == 0) sh.count = 0;
   __syncthreads();
@@ -315,29 +377,40 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
   // ---- the span's top-k
   rank_keys(sh.cand, M, k, sh.list, tid);
   // the span's (max, sum) from the warps'
-  float m_cta = -INFINITY, s_cta = 0.f;
+  float m_cta = -INFINITY, s_cta = 0.f, t_cta = 0.f;
   if (warp == 0) {
     float mw = lane < kWarps ? sh.warp_ms[lane].x : -INFINITY;
     float sw = lane < kWarps ? sh.warp_ms[lane].y : 0.f;
+    float tw = 0.f;
+    if constexpr (ENT) tw = lane < kWarps ? sh.warp_t[lane] : 0.f;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
       const float m_o = __shfl_xor_sync(kFull, mw, off);
       const float s_o = __shfl_xor_sync(kFull, sw, off);
-      merge_ms(mw, sw, m_o, s_o);
+      if constexpr (ENT) {
+        const float t_o = __shfl_xor_sync(kFull, tw, off);
+        merge_mst(mw, sw, tw, m_o, s_o, t_o);
+      } else {
+        merge_ms(mw, sw, m_o, s_o);
+      }
     }
     m_cta = mw;
     s_cta = sw;
+    t_cta = tw;
   }
   __syncthreads();
   const int got = M < k ? M : k;
 
   // ---- combine the spans of the row in the leader CTA
-  float m_row = m_cta, s_row = s_cta;
+  float m_row = m_cta, s_row = s_cta, t_row = t_cta;
   if (a.parts > 1) {
     cg::cluster_group cluster = cg::this_cluster();
     Smem* leader = cluster.map_shared_rank(&sh, 0);
     if (tid < k) leader->part[part][tid] = tid < got ? sh.list[tid] : 0ull;
-    if (tid == 0) leader->part_ms[part] = make_float2(m_cta, s_cta);
+    if (tid == 0) {
+      leader->part_ms[part] = make_float2(m_cta, s_cta);
+      if constexpr (ENT) leader->part_t[part] = t_cta;
+    }
     cluster.sync();
     if (part != 0) return;
     // the parts' keys: zeros (fewer than k in a span) rank below every real key and
@@ -347,14 +420,22 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
     if (warp == 0) {
       float mw = lane < a.parts ? sh.part_ms[lane].x : -INFINITY;
       float sw = lane < a.parts ? sh.part_ms[lane].y : 0.f;
+      float tw = 0.f;
+      if constexpr (ENT) tw = lane < a.parts ? sh.part_t[lane] : 0.f;
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) {
         const float m_o = __shfl_xor_sync(kFull, mw, off);
         const float s_o = __shfl_xor_sync(kFull, sw, off);
-        merge_ms(mw, sw, m_o, s_o);
+        if constexpr (ENT) {
+          const float t_o = __shfl_xor_sync(kFull, tw, off);
+          merge_mst(mw, sw, tw, m_o, s_o, t_o);
+        } else {
+          merge_ms(mw, sw, m_o, s_o);
+        }
       }
       m_row = mw;
       s_row = sw;
+      t_row = tw;
     }
     __syncthreads();
     rank_keys(sh.cand, P, k, sh.list, tid);
@@ -372,10 +453,20 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
       a.topk_logq[static_cast<size_t>(row) * k + lane] = (key_value(key) - mx) - logs;
     }
     if (lane == 0 && a.lse) a.lse[row] = mx + logs;
+    if constexpr (ENT) {
+      if (lane == 0) {
+        // H = -Σ q ln q = ln s - ln2 (t / s); q ln q -> 0 where q underflows.  H >= 0
+        // exactly; rounding can take a near-one-hot row a hair below, so clamp (this
+        // also keeps lambda_d >= 0, as the tree build requires)
+        const float H = fmaxf(logs - 0.6931471805599453f * __fdiv_rn(t_row, s_row), 0.f);
+        if (a.entropy) a.entropy[row] = H;
+        if (a.lambda_d) a.lambda_d[row] = __fdiv_rn(__fmul_rn(a.beta, H), __fadd_rn(H, a.C));
+      }
+    }
   }
 }
 
-template <typename T, int VMAX>
+template <typename T, int VMAX, bool ENT>
 int max_active_clusters(int parts) {
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(parts));
@@ -388,41 +479,45 @@ int max_active_clusters(int parts) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, topk_kernel<T, VMAX>, &cfg) != cudaSuccess) {
+  if (cudaOccupancyMaxActiveClusters(&n, topk_kernel<T, VMAX, ENT>, &cfg) != cudaSuccess) {
     cudaGetLastError();
     return 0;
   }
   return n;
 }
 
-// Resident clusters of `parts` CTAs for the kernel of element size eb and register
-// bound vmax, queried once per device.
-int active_clusters(int eb, int vmax, int parts) {
+template <bool ENT>
+int max_active_clusters_of(int eb, int vmax, int parts) {
+  if (eb == 4)
+    return vmax == 4 ? max_active_clusters<float, 4, ENT>(parts)
+           : vmax == 8 ? max_active_clusters<float, 8, ENT>(parts)
+                       : max_active_clusters<float, 16, ENT>(parts);
+  return vmax == 4 ? max_active_clusters<__nv_bfloat16, 4, ENT>(parts)
+         : vmax == 8 ? max_active_clusters<__nv_bfloat16, 8, ENT>(parts)
+                     : max_active_clusters<__nv_bfloat16, 16, ENT>(parts);
+}
+
+// Resident clusters of `parts` CTAs for the kernel of element size eb, register
+// bound vmax and entropy flag ent, queried once per device.
+int active_clusters(int eb, int vmax, int parts, bool ent) {
   static std::mutex mu;
-  static int cache[64][2][3][kMaxParts + 1];
-  static bool done[64][2][3][kMaxParts + 1];
+  static int cache[64][2][3][2][kMaxParts + 1];
+  static bool done[64][2][3][2][kMaxParts + 1];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
-  const int ti = eb == 4 ? 0 : 1, vi = vmax == 4 ? 0 : (vmax == 8 ? 1 : 2);
+  const int ti = eb == 4 ? 0 : 1, vi = vmax == 4 ? 0 : (vmax == 8 ? 1 : 2), ei = ent ? 1 : 0;
   std::lock_guard<std::mutex> lock(mu);
-  if (!done[dev][ti][vi][parts]) {
-    int n;
-    if (eb == 4)
-      n = vmax == 4 ? max_active_clusters<float, 4>(parts)
-          : vmax == 8 ? max_active_clusters<float, 8>(parts) : max_active_clusters<float, 16>(parts);
-    else
-      n = vmax == 4 ? max_active_clusters<__nv_bfloat16, 4>(parts)
-          : vmax == 8 ? max_active_clusters<__nv_bfloat16, 8>(parts)
-                      : max_active_clusters<__nv_bfloat16, 16>(parts);
-    cache[dev][ti][vi][parts] = n;
-    done[dev][ti][vi][parts] = true;
+  if (!done[dev][ti][vi][ei][parts]) {
+    cache[dev][ti][vi][ei][parts] = ent ? max_active_clusters_of<true>(eb, vmax, parts)
+                                        : max_active_clusters_of<false>(eb, vmax, parts);
+    done[dev][ti][vi][ei][parts] = true;
   }
-  return cache[dev][ti][vi][parts];
+  return cache[dev][ti][vi][ei][parts];
 }
 
 // Spans per row (= cluster size) and vectors per thread: the estimated time is
 // waves of resident clusters x (fixed cost + cost per vector per thread).
-Plan make_plan(int B, int L, int V, int elem_bytes) {
+Plan make_plan(int B, int L, int V, int elem_bytes, bool ent) {
   Plan p;
   p.rows = B * L;
   p.epv = 16 / elem_bytes;
@@ -435,7 +530,7 @@ Plan make_plan(int B, int L, int V, int elem_bytes) {
     if (vpt > 16) continue;
     if (parts > 1 && (nvec + vpt * kThreads - 1) / (vpt * kThreads) < parts) continue;  // empty span
     const int vmax = vpt <= 4 ? 4 : (vpt <= 8 ? 8 : 16);
-    int act = active_clusters(elem_bytes, vmax, parts);
+    int act = active_clusters(elem_bytes, vmax, parts, ent);
     if (act < 1) act = parts == 1 ? sm_count() : 0;
     if (act < 1) continue;
     const double waves = std::ceil(static_cast<double>(p.rows) / act);
@@ -450,7 +545,7 @@ Plan make_plan(int B, int L, int V, int elem_bytes) {
   return p;
 }
 
-template <typename T, int VMAX>
+template <typename T, int VMAX, bool ENT>
 cudaError_t launch(const Plan& p, const Args& a, cudaStream_t stream) {
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(p.rows) * p.parts);
@@ -464,7 +559,51 @@ cudaError_t launch(const Plan& p, const Args& a, cudaStream_t stream) {
   attr[1] = pdl_attribute();
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, topk_kernel<T, VMAX>, a);
+  return cudaLaunchKernelEx(&cfg, topk_kernel<T, VMAX, ENT>, a);
+}
+
+template <bool ENT>
+cudaError_t dispatch(int dtype, const Plan& p, const Args& a, cudaStream_t stream) {
+  if (dtype == PRESTO_F32)
+    return p.vmax == 4 ? launch<float, 4, ENT>(p, a, stream)
+           : p.vmax == 8 ? launch<float, 8, ENT>(p, a, stream)
+                         : launch<float, 16, ENT>(p, a, stream);
+  return p.vmax == 4 ? launch<__nv_bfloat16, 4, ENT>(p, a, stream)
+         : p.vmax == 8 ? launch<__nv_bfloat16, 8, ENT>(p, a, stream)
+                       : launch<__nv_bfloat16, 16, ENT>(p, a, stream);
+}
+
+// Checks and launch shared by presto_topk and presto_topk_entropy.
+int topk_common(const void* logits, int dtype, int B, int L, int V, long long row_stride, int k,
+                int32_t* topk_ids, float* topk_logq, float* lse, float* entropy, float* lambda_d,
+                float beta, float C, int32_t* dev_status, cudaStream_t stream) {
+  PRESTO_CHECK_ARG(logits && topk_ids && topk_logq);
+  PRESTO_CHECK_ARG(dtype == PRESTO_F32 || dtype == PRESTO_BF16);
+  PRESTO_CHECK_ARG(B >= 1 && L >= 1 && V >= 1 && k >= 1 && row_stride >= V);
+  PRESTO_CHECK_ARG(k <= V);
+  PRESTO_CHECK_LIMIT(k <= kMaxK && V < kMaxV && L <= kMaxL);
+  const int eb = dtype == PRESTO_F32 ? 4 : 2;
+  PRESTO_CHECK_ARG(reinterpret_cast<uintptr_t>(logits) % eb == 0);
+  const bool ent = entropy || lambda_d;
+  const Plan p = make_plan(B, L, V, eb, ent);
+  Args a;
+  a.logits = logits;
+  a.row_stride = row_stride;
+  a.V = V;
+  a.k = k;
+  a.parts = p.parts;
+  a.vpt = p.vpt;
+  a.topk_ids = topk_ids;
+  a.topk_logq = topk_logq;
+  a.lse = lse;
+  a.entropy = entropy;
+  a.lambda_d = lambda_d;
+  a.beta = beta;
+  a.C = C;
+  a.dev_status = dev_status;
+  const cudaError_t e = ent ? dispatch<true>(dtype, p, a, stream) : dispatch<false>(dtype, p, a, stream);
+  if (e != cudaSuccess) return PRESTO_ERR_CUDA;
+  return launch_status();
 }
 
 }  // namespace
@@ -482,37 +621,23 @@ extern "C" int presto_topk(const void* logits, int dtype, int B, int L, int V,
                            long long row_stride, int k, int32_t* topk_ids, float* topk_logq,
                            float* lse, void* ws, size_t ws_bytes, int32_t* dev_status,
                            presto_stream_t stream) {
-  PRESTO_CHECK_ARG(logits && topk_ids && topk_logq);
-  PRESTO_CHECK_ARG(dtype == PRESTO_F32 || dtype == PRESTO_BF16);
-  PRESTO_CHECK_ARG(B >= 1 && L >= 1 && V >= 1 && k >= 1 && row_stride >= V);
-  PRESTO_CHECK_ARG(k <= V);
-  PRESTO_CHECK_LIMIT(k <= kMaxK && V < kMaxV && L <= kMaxL);
   (void)ws;
   (void)ws_bytes;
-  const int eb = dtype == PRESTO_F32 ? 4 : 2;
-  PRESTO_CHECK_ARG(reinterpret_cast<uintptr_t>(logits) % eb == 0);
-  const Plan p = make_plan(B, L, V, eb);
-  Args a;
-  a.logits = logits;
-  a.row_stride = row_stride;
-  a.V = V;
-  a.k = k;
-  a.parts = p.parts;
-  a.vpt = p.vpt;
-  a.topk_ids = topk_ids;
-  a.topk_logq = topk_logq;
-  a.lse = lse;
-  a.dev_status = dev_status;
-  cudaError_t e;
-  if (dtype == PRESTO_F32)
-    e = p.vmax == 4 ? launch<float, 4>(p, a, stream)
-        : p.vmax == 8 ? launch<float, 8>(p, a, stream) : launch<float, 16>(p, a, stream);
-  else
-    e = p.vmax == 4 ? launch<__nv_bfloat16, 4>(p, a, stream)
-        : p.vmax == 8 ? launch<__nv_bfloat16, 8>(p, a, stream)
-                      : launch<__nv_bfloat16, 16>(p, a, stream);
-  if (e != cudaSuccess) return PRESTO_ERR_CUDA;
-  return launch_status();
+  return topk_common(logits, dtype, B, L, V, row_stride, k, topk_ids, topk_logq, lse, nullptr,
+                     nullptr, 0.f, 0.f, dev_status, stream);
+}
+
+extern "C" int presto_topk_entropy(const void* logits, int dtype, int B, int L, int V,
+                                   long long row_stride, int k, float beta, float C,
+                                   int32_t* topk_ids, float* topk_logq, float* lse,
+                                   float* entropy, float* lambda_d, void* ws, size_t ws_bytes,
+                                   int32_t* dev_status, presto_stream_t stream) {
+  (void)ws;
+  (void)ws_bytes;
+  PRESTO_CHECK_ARG(entropy || lambda_d);
+  if (lambda_d) PRESTO_CHECK_ARG(beta > 0.f && beta < INFINITY && C > 0.f && C < INFINITY);
+  return topk_common(logits, dtype, B, L, V, row_stride, k, topk_ids, topk_logq, lse, entropy,
+                     lambda_d, beta, C, dev_status, stream);
 }
 
 // ---------------------------------------------------------------------------

@@ -99,7 +99,7 @@ def path_score64(ids_b, logq_b, ctx_b, table, miss, lam, path):
         rho = None
         if table is not None:
             rho = table.get(O.trigram_context(ctx_b, path[: d - 1]) + (path[d - 1],), miss)
-        S += O.token_score(logq_b[d - 1, j], rho, lam, "fp64")
+        S += O.token_score(logq_b[d - 1, j], rho, O._lam_at(lam, d - 1), "fp64")
     return S
 
 
@@ -114,7 +114,7 @@ def assert_tree_close(g, ids, logq, ctx, table, miss, lam, N, tol=LOGQ_TOL):
         assert int(g["n_nodes"][b]) == n
         gp = [path_of(g["token"][b], g["parent"][b], i) for i in range(n)]
         op = [path_of(o["token"][b], o["parent"][b], i) for i in range(n)]
-        gS = [path_score64(ids[b], logq[b], ctx[b], table, miss, lam, p) for p in gp]
+        gS = [path_score64(ids[b], logq[b], ctx[b], table, miss, O._lam_of(lam, b), p) for p in gp]
         err = rel_close(g["score"][b][:n], gS)
         assert err <= tol, (b, err)
         assert all(gS[i + 1] <= gS[i] + tol * max(1, abs(gS[i])) for i in range(n - 1))

@@ -531,6 +531,55 @@ def accept(node_token, node_parent, n_nodes, target_token, L):
     return acc, path_out, bonus
 
 
+# ---------------------------------------------------------------------------
+# Step 7 (self-speculative rounds, App. C (II)): the next round's drafter rows are
+# the mask slots attached to the end of the accepted path; the slots of every
+# other node (rejected branches) are discarded.
+# ---------------------------------------------------------------------------
+
+def accepted_node(accept_len, accept_path):
+    """a*_b = accept_path[b, accept_len[b]]: the deepest accepted node (node 0, the
+    root, when nothing was accepted)."""
+    accept_len = np.asarray(accept_len)
+    accept_path = np.asarray(accept_path)
+    out = np.empty(len(accept_len), np.int64)
+    for b, n in enumerate(accept_len):
+        if not 0 <= int(n) < accept_path.shape[1]:
+            raise ValueError("accept_len outside the path")
+        out[b] = int(accept_path[b, int(n)])
+    return out
+
+
+def accepted_slot_rows(slot_logits, accept_len, accept_path, slot_offset, L):
+    """slot_logits [B, n_prev, n_slots, V]: the logits the self-speculative forward
+    produced at the mask slots of each previous-round node.  Returns [B, L, V]:
+    row j of sequence b is slot slot_offset + j of a*_b, so the slot that predicts
+    the token at depth j + 1 of the next tree feeds drafter row j (slot_offset is
+    the model's distance between a node and the slot of the position after the
+    bonus token)."""
+    x = np.asarray(slot_logits)
+    B, n_prev, n_slots, V = x.shape
+    if not (0 <= slot_offset and slot_offset + L <= n_slots):
+        raise ValueError("slots slot_offset .. slot_offset + L - 1 must exist")
+    a = accepted_node(accept_len, accept_path)
+    rows = np.empty((B, L, V), x.dtype)
+    for b in range(B):
+        if not 0 <= a[b] < n_prev:
+            raise ValueError("accepted node outside the previous tree")
+        for j in range(L):
+            rows[b, j] = x[b, a[b], slot_offset + j]
+    return rows
+
+
+def next_context(node_token, accept_len, accept_path, bonus):
+    """The last two committed tokens after acceptance, the next round's ctx2: the
+    token of a*_b and the bonus token (App. C (I): the position after the last
+    accepted token holds the model's own prediction).  [B, 2] int64."""
+    node_token = np.asarray(node_token)
+    a = accepted_node(accept_len, accept_path)
+    return np.array([[int(node_token[b, a[b]]), int(bonus[b])] for b in range(len(a))], np.int64)
+
+
 def coverage_bound(target_fn, topk_sets, L):
     """Obs. 1 (§3): follow the target's greedy continuation and count the longest
     prefix whose token at each depth d lies in the depth-d candidate set.

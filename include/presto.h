@@ -6,6 +6,8 @@
  *
  *   presto_topk             per-position log-softmax and top-k of the drafter logits
  *   presto_topk_entropy     the same, plus each row's entropy and adaptive lambda_d
+ *   presto_topk_slots       the same over the mask slots of the accepted node
+ *                           (self-speculative rounds)
  *   presto_score_build_tree prefix-aligned scores + best-first tree up to N nodes
  *                           (_ex: beam search / printed Alg. 2, per-position lambda)
  *   presto_tree_mask        ancestor bitmask and position ids of the tree tokens
@@ -67,6 +69,7 @@ typedef struct CUstream_st* presto_stream_t;  /* same type as cudaStream_t */
 #define PRESTO_DEV_DUP_SIBLING 0x40   /* two candidates of one position share a token */
 #define PRESTO_DEV_TABLE_FULL 0x80    /* n-gram insert found no free slot         */
 #define PRESTO_DEV_NONFINITE 0x100    /* a logits row has no finite maximum       */
+#define PRESTO_DEV_BAD_PATH 0x200     /* accept_len / accept_path entry out of range */
 
 /* ---- element types -------------------------------------------------------- */
 #define PRESTO_F32 0
@@ -145,6 +148,43 @@ int presto_topk_entropy(const void* logits, int dtype, int B, int L, int V,
                         long long row_stride, int k, float beta, float C, int32_t* topk_ids,
                         float* topk_logq, float* lse, float* entropy, float* lambda_d, void* ws,
                         size_t ws_bytes, int32_t* dev_status, presto_stream_t stream);
+
+/*
+ * presto_topk_slots - presto_topk over the mask slots of the accepted path, for
+ * self-speculative rounds (App. C (II)): one forward of the dLLM verified the
+ * previous tree and denoised a block of mask slots attached to every one of its
+ * nodes; only the slots of the deepest accepted node a*_b stay valid, and they are
+ * the next round's drafter rows.
+ *
+ *   slot_logits  [B, n_prev, n_slots, row_stride] dtype PRESTO_F32 or PRESTO_BF16:
+ *                the logits at slot j of node i of sequence b (first V entries
+ *                of a row are read).  Only the rows named below are read; the
+ *                slots of every other node are never touched.
+ *   accept_len, accept_path  [B], [B, path_len] int32, as written by presto_accept
+ *                (path_len = its L + 1): a*_b = accept_path[b][accept_len[b]].
+ *                Read on the device after the kernel before this one on `stream`
+ *                finishes, so presto_accept may run just before with no host sync.
+ *   slot_offset, L  drafter row j (depth j + 1 of the next tree) is slot
+ *                slot_offset + j of a*_b; 0 <= slot_offset <= n_slots - L.  Which
+ *                slot holds the position after the bonus token depends on the model
+ *                (the paper does not fix it): 1 when slot j of a node predicts the
+ *                token j + 1 places after it, since the bonus takes the first place.
+ *   node_token, bonus, ctx2_next  nullable together: [B, n_prev], [B] int32 in
+ *                (presto_score_build_tree's node_token and presto_accept's bonus),
+ *                [B, 2] int32 out = (node_token[b][a*_b], bonus[b]), the last two
+ *                committed tokens, i.e. the next round's ctx2.  Must not alias the
+ *                inputs.
+ *   topk_ids, topk_logq, lse, ws, dev_status  as presto_topk with B x L rows.
+ *                PRESTO_DEV_BAD_PATH when accept_len[b] is outside [0, path_len) or
+ *                the node it selects is outside [0, n_prev); that sequence then
+ *                reads the root's slots.
+ */
+int presto_topk_slots(const void* slot_logits, int dtype, int B, int n_prev, int n_slots, int V,
+                      long long row_stride, const int32_t* accept_len,
+                      const int32_t* accept_path, int path_len, int slot_offset, int L, int k,
+                      const int32_t* node_token, const int32_t* bonus, int32_t* ctx2_next,
+                      int32_t* topk_ids, float* topk_logq, float* lse, void* ws, size_t ws_bytes,
+                      int32_t* dev_status, presto_stream_t stream);
 
 /*
  * Trigram prefix signal rho_d(t | t_{d-2}, t_{d-1}) (§4.1; the paper instantiates

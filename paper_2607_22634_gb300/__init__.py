@@ -24,6 +24,7 @@ from ._lib import (  # noqa: F401
     presto_topk,
     presto_topk_entropy,
     presto_topk_noalloc,
+    presto_topk_slots,
     presto_topk_workspace,
     presto_tree_attention,
     presto_tree_mask,

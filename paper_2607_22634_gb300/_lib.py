@@ -26,7 +26,7 @@ NGRAM3_EMPTY = 0xFFFFFFFFFFFFFFFF
 DEV_STATUS_BITS = {
     0x1: "BAD_PARENT", 0x2: "BAD_TOKEN", 0x4: "BAD_KVLEN", 0x8: "BAD_NNODES",
     0x10: "POSITIVE_SCORE", 0x20: "TIMEOUT", 0x40: "DUP_SIBLING", 0x80: "TABLE_FULL",
-    0x100: "NONFINITE",
+    0x100: "NONFINITE", 0x200: "BAD_PATH",
 }
 
 
@@ -48,6 +48,8 @@ _SIGS = {
     "presto_topk": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, _P, _P, _P, _P,
                          ctypes.c_size_t, _P, _P]),
     "presto_topk_noalloc": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, _P, _P, _P, _P, _P]),
+    "presto_topk_slots": (_I, [_P, _I, _I, _I, _I, _I, ctypes.c_longlong, _P, _P, _I, _I, _I, _I,
+                               _P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "presto_topk_entropy": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, ctypes.c_float,
                                  ctypes.c_float, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "presto_ngram3_clear": (_I, [ctypes.POINTER(Ngram3), _P]),
@@ -212,6 +214,49 @@ def presto_topk_entropy(logits, k, beta=None, C=None, topk_ids=None, topk_logq=N
                                     _ptr(dev_status), _stream(stream))
     _check(st, "presto_topk_entropy")
     return topk_ids, topk_logq, lse, entropy, lambda_d
+
+
+def presto_topk_slots(slot_logits, accept_len, accept_path, slot_offset, L, k, node_token=None,
+                      bonus=None, ctx2_next=None, topk_ids=None, topk_logq=None, lse=None, ws=None,
+                      dev_status=None, stream=None, with_lse=True):
+    """Top-k of the next round's drafter rows, read in place from the mask slots of
+    the deepest accepted node (App. C (II)).  slot_logits [B, n_prev, n_slots, V]
+    (unit last stride, packed); accept_len [B], accept_path [B, path_len] from
+    presto_accept.  With node_token and bonus also returns ctx2_next [B, 2].
+    Returns (topk_ids, topk_logq, lse, ctx2_next)."""
+    if slot_logits.dim() != 4 or slot_logits.stride(3) != 1:
+        raise ValueError("slot_logits must be [B, n_prev, n_slots, V] with unit last stride")
+    B, n_prev, n_slots, V = slot_logits.shape
+    rs = slot_logits.stride(2)
+    if slot_logits.stride(1) != n_slots * rs or slot_logits.stride(0) != n_prev * n_slots * rs:
+        raise ValueError("slot_logits rows must be packed")
+    dtype = {torch.float32: PRESTO_F32, torch.bfloat16: PRESTO_BF16}.get(slot_logits.dtype)
+    if dtype is None:
+        raise ValueError("slot_logits must be float32 or bfloat16")
+    dev = slot_logits.device
+    path_len = accept_path.shape[1]
+    _need(accept_len, torch.int32, (B,), "accept_len")
+    _need(accept_path, torch.int32, (B, path_len), "accept_path")
+    topk_ids = torch.empty(B, L, k, dtype=torch.int32, device=dev) if topk_ids is None else topk_ids
+    topk_logq = torch.empty(B, L, k, dtype=torch.float32, device=dev) if topk_logq is None else topk_logq
+    if lse is None and with_lse:
+        lse = torch.empty(B, L, dtype=torch.float32, device=dev)
+    if node_token is not None:
+        _need(node_token, torch.int32, (B, n_prev), "node_token")
+        _need(bonus, torch.int32, (B,), "bonus")
+        if ctx2_next is None:
+            ctx2_next = torch.empty(B, 2, dtype=torch.int32, device=dev)
+        _need(ctx2_next, torch.int32, (B, 2), "ctx2_next")
+    _need(topk_ids, torch.int32, (B, L, k), "topk_ids")
+    _need(topk_logq, torch.float32, (B, L, k), "topk_logq")
+    ws, nws = _ws(presto_topk_workspace(B, L, V, k), dev, ws)
+    st = load().presto_topk_slots(_ptr(slot_logits), dtype, B, n_prev, n_slots, V, rs,
+                                  _ptr(accept_len), _ptr(accept_path), path_len, slot_offset, L, k,
+                                  _ptr(node_token), _ptr(bonus), _ptr(ctx2_next), _ptr(topk_ids),
+                                  _ptr(topk_logq), _ptr(lse), _ptr(ws), nws, _ptr(dev_status),
+                                  _stream(stream))
+    _check(st, "presto_topk_slots")
+    return topk_ids, topk_logq, lse, ctx2_next
 
 
 # ------------------------------------------------------------------ trigram table

@@ -23,6 +23,10 @@
 //     s = Σ 2^u, u = x log2e - max2, each thread sums t = Σ 2^u u, and the merges
 //     carry t along (when the reference maximum drops by δ, t -> 2^δ (t + δ s)).
 //     Then H = ln s - ln2 t / s, and lambda_d = beta H / (H + C).
+//   * With slot rows (self-speculative rounds, App. C (II)) row j of sequence b is
+//     read in place from slot slot_off + j of the deepest accepted node a*_b =
+//     accept_path[b][accept_len[b]], looked up on the device after the accept
+//     kernel that precedes it on the stream: no gather copy, no host round trip.
 #include <cuda_bf16.h>
 
 #include <cooperative_groups.h>
@@ -152,8 +156,39 @@ struct Args {
   float* entropy;   // ENT: [rows] H in nats, nullable
   float* lambda_d;  // ENT: [rows] beta H / (H + C), nullable
   float beta, C;
+  // slot rows (acc_len non-null): logits = [B][n_prev][n_slots][row_stride]
+  const int32_t* acc_len;    // [B]
+  const int32_t* acc_path;   // [B][path_len]
+  int path_len, n_prev, n_slots, slot_off, Lrows;
+  const int32_t* node_token;  // [B][n_prev], nullable (with bonus, ctx2_next)
+  const int32_t* bonus;       // [B]
+  int32_t* ctx2_next;         // [B][2]
   int32_t* dev_status;
 };
+
+// Row `row` of the launch: a plain row of the logits, or (slot rows) slot
+// slot_off + j of the accepted node of sequence b, row = b * Lrows + j.  Slot rows
+// read the accept results, so the caller has passed the grid dependency wait.  A
+// path entry out of range is reported and reads the root's slots instead.
+template <typename T>
+__device__ __forceinline__ const T* row_base(const Args& a, int row, bool first) {
+  const T* base = static_cast<const T*>(a.logits);
+  if (!a.acc_len) return base + static_cast<long long>(row) * a.row_stride;
+  const int b = row / a.Lrows, j = row - b * a.Lrows;
+  const int len = a.acc_len[b];
+  int node = -1;
+  if (len >= 0 && len < a.path_len) node = a.acc_path[static_cast<long long>(b) * a.path_len + len];
+  if (node < 0 || node >= a.n_prev) {
+    if (first) report(a.dev_status, PRESTO_DEV_BAD_PATH);
+    node = 0;
+  }
+  if (first && j == 0 && a.ctx2_next) {
+    a.ctx2_next[2 * b] = a.node_token[static_cast<long long>(b) * a.n_prev + node];
+    a.ctx2_next[2 * b + 1] = a.bonus[b];
+  }
+  const long long slot = (static_cast<long long>(b) * a.n_prev + node) * a.n_slots + a.slot_off + j;
+  return base + slot * a.row_stride;
+}
 
 struct Smem {
   unsigned long long cand[kCandCap];
@@ -194,7 +229,8 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
   const int part = blockIdx.x % a.parts;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int k = a.k, V = a.V;
-  const T* rowp = static_cast<const T*>(a.logits) + static_cast<long long>(row) * a.row_stride;
+  if (a.acc_len) pdl_wait();  // slot rows: the accept results come from the previous kernel
+  const T* rowp = row_base<T>(a, row, part == 0 && tid == 0);
   // the row's 16-byte-aligned vectors [head, head + nvec * n); the few elements
   // before and after are read one by one
   const int mis = static_cast<int>(reinterpret_cast<uintptr_t>(rowp) & 15);
@@ -573,10 +609,22 @@ cudaError_t dispatch(int dtype, const Plan& p, const Args& a, cudaStream_t strea
                        : launch<__nv_bfloat16, 16, ENT>(p, a, stream);
 }
 
-// Checks and launch shared by presto_topk and presto_topk_entropy.
+// Slot-row source of presto_topk_slots (see Args).
+struct SlotRows {
+  const int32_t* acc_len;
+  const int32_t* acc_path;
+  int path_len, n_prev, n_slots, slot_off;
+  const int32_t* node_token;
+  const int32_t* bonus;
+  int32_t* ctx2_next;
+};
+
+// Checks and launch shared by presto_topk, presto_topk_entropy and presto_topk_slots
+// (B x L output rows; `slots` null: row r of the logits is output row r).
 int topk_common(const void* logits, int dtype, int B, int L, int V, long long row_stride, int k,
                 int32_t* topk_ids, float* topk_logq, float* lse, float* entropy, float* lambda_d,
-                float beta, float C, int32_t* dev_status, cudaStream_t stream) {
+                float beta, float C, const SlotRows* slots, int32_t* dev_status,
+                cudaStream_t stream) {
   PRESTO_CHECK_ARG(logits && topk_ids && topk_logq);
   PRESTO_CHECK_ARG(dtype == PRESTO_F32 || dtype == PRESTO_BF16);
   PRESTO_CHECK_ARG(B >= 1 && L >= 1 && V >= 1 && k >= 1 && row_stride >= V);
@@ -586,7 +634,7 @@ int topk_common(const void* logits, int dtype, int B, int L, int V, long long ro
   PRESTO_CHECK_ARG(reinterpret_cast<uintptr_t>(logits) % eb == 0);
   const bool ent = entropy || lambda_d;
   const Plan p = make_plan(B, L, V, eb, ent);
-  Args a;
+  Args a{};
   a.logits = logits;
   a.row_stride = row_stride;
   a.V = V;
@@ -600,6 +648,18 @@ int topk_common(const void* logits, int dtype, int B, int L, int V, long long ro
   a.lambda_d = lambda_d;
   a.beta = beta;
   a.C = C;
+  if (slots) {
+    a.acc_len = slots->acc_len;
+    a.acc_path = slots->acc_path;
+    a.path_len = slots->path_len;
+    a.n_prev = slots->n_prev;
+    a.n_slots = slots->n_slots;
+    a.slot_off = slots->slot_off;
+    a.Lrows = L;
+    a.node_token = slots->node_token;
+    a.bonus = slots->bonus;
+    a.ctx2_next = slots->ctx2_next;
+  }
   a.dev_status = dev_status;
   const cudaError_t e = ent ? dispatch<true>(dtype, p, a, stream) : dispatch<false>(dtype, p, a, stream);
   if (e != cudaSuccess) return PRESTO_ERR_CUDA;
@@ -624,7 +684,7 @@ extern "C" int presto_topk(const void* logits, int dtype, int B, int L, int V,
   (void)ws;
   (void)ws_bytes;
   return topk_common(logits, dtype, B, L, V, row_stride, k, topk_ids, topk_logq, lse, nullptr,
-                     nullptr, 0.f, 0.f, dev_status, stream);
+                     nullptr, 0.f, 0.f, nullptr, dev_status, stream);
 }
 
 extern "C" int presto_topk_entropy(const void* logits, int dtype, int B, int L, int V,
@@ -637,7 +697,28 @@ extern "C" int presto_topk_entropy(const void* logits, int dtype, int B, int L, 
   PRESTO_CHECK_ARG(entropy || lambda_d);
   if (lambda_d) PRESTO_CHECK_ARG(beta > 0.f && beta < INFINITY && C > 0.f && C < INFINITY);
   return topk_common(logits, dtype, B, L, V, row_stride, k, topk_ids, topk_logq, lse, entropy,
-                     lambda_d, beta, C, dev_status, stream);
+                     lambda_d, beta, C, nullptr, dev_status, stream);
+}
+
+extern "C" int presto_topk_slots(const void* slot_logits, int dtype, int B, int n_prev,
+                                 int n_slots, int V, long long row_stride,
+                                 const int32_t* accept_len, const int32_t* accept_path,
+                                 int path_len, int slot_offset, int L, int k,
+                                 const int32_t* node_token, const int32_t* bonus,
+                                 int32_t* ctx2_next, int32_t* topk_ids, float* topk_logq,
+                                 float* lse, void* ws, size_t ws_bytes, int32_t* dev_status,
+                                 presto_stream_t stream) {
+  (void)ws;
+  (void)ws_bytes;
+  PRESTO_CHECK_ARG(accept_len && accept_path);
+  PRESTO_CHECK_ARG(B >= 1 && n_prev >= 1 && n_slots >= 1 && path_len >= 1 && L >= 1);
+  PRESTO_CHECK_ARG(slot_offset >= 0 && slot_offset <= n_slots - L);
+  PRESTO_CHECK_ARG((node_token && bonus && ctx2_next) || (!node_token && !bonus && !ctx2_next));
+  PRESTO_CHECK_LIMIT(static_cast<long long>(B) * n_prev * n_slots < (1ll << 31));
+  const SlotRows sr{accept_len, accept_path, path_len, n_prev, n_slots, slot_offset,
+                    node_token, bonus, ctx2_next};
+  return topk_common(slot_logits, dtype, B, L, V, row_stride, k, topk_ids, topk_logq, lse,
+                     nullptr, nullptr, 0.f, 0.f, &sr, dev_status, stream);
 }
 
 // ---------------------------------------------------------------------------

@@ -44,6 +44,8 @@ def parse_args(argv=None):
     p.add_argument("--e2e-steps", type=int, default=2000)
     p.add_argument("--cpu-seconds", type=float, default=15.0)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-variants", action="store_true",
+                   help="skip timing the search policies, adaptive lambda and slot top-k")
     p.add_argument("--oracle-worker", action="store_true", help=argparse.SUPPRESS)
     return p.parse_args(argv)
 
@@ -244,6 +246,81 @@ def profiled_traffic(kernel):
     return rec.get("dram_bytes_per_launch")
 
 
+def time_variants(args, P, w, step, sets, side, ngram):
+    import torch
+    dev = step.device
+    B, L, k, N = w.B, w.L, w.k, w.N
+    f32, i32 = torch.float32, torch.int32
+    lam_d = torch.full((B, L), w.lam, dtype=f32, device=dev)
+    ent = torch.empty(B, L, dtype=f32, device=dev)
+    lam_out = torch.empty(B, L, dtype=f32, device=dev)
+    ws_b = torch.empty(max(P.presto_build_workspace(B, L, k, N, 10), 256), dtype=torch.uint8,
+                       device=dev)
+    tree = {key: torch.empty_like(v) for key, v in step.tree.items()}
+    # slot logits of every node of the tree: [B, N, L + 1, V]; set s accepts node
+    # 1 + s (mod N - 1) of every sequence, so each launch reads other rows
+    esz = sets[0]["logits"].element_size()
+    slots = None
+    if B * N * (L + 1) * w.V * esz <= (4 << 30):
+        g = torch.Generator(device=dev)
+        g.manual_seed(w.seed + 77)
+        slots = torch.randn(B, N, L + 1, w.V, generator=g, device=dev).to(sets[0]["logits"].dtype)
+        acc_len = torch.ones(B, dtype=i32, device=dev)
+        paths = []
+        for s in range(len(sets)):
+            pth = torch.full((B, L + 1), -1, dtype=i32, device=dev)
+            pth[:, 0] = 0
+            pth[:, 1] = 1 + s % max(1, N - 1)
+            paths.append(pth)
+    calls = {
+        "build_beam10": lambda st, s, i: P.presto_score_build_tree(
+            step.topk_ids, step.topk_logq, st["ctx"], ngram, w.lam, N, b=w.branching,
+            out=tree, ws=ws_b, stream=s, policy=P.SEARCH_BEAM, beam_width=10),
+        "build_eager": lambda st, s, i: P.presto_score_build_tree(
+            step.topk_ids, step.topk_logq, st["ctx"], ngram, w.lam, N, b=w.branching,
+            out=tree, ws=ws_b, stream=s, policy=P.SEARCH_EAGER),
+        "build_lambda_d": lambda st, s, i: P.presto_score_build_tree(
+            step.topk_ids, step.topk_logq, st["ctx"], ngram, w.lam, N, b=w.branching,
+            out=tree, ws=ws_b, stream=s, lambda_d=lam_d),
+        "topk_entropy": lambda st, s, i: P.presto_topk_entropy(
+            st["logits"], k, 0.5, 2.0, step.topk_ids, step.topk_logq, step.lse, ent, lam_out,
+            ws=step.ws_topk, stream=s),
+    }
+    if slots is not None:
+        calls["topk_slots"] = lambda st, s, i: P.presto_topk_slots(
+            slots, acc_len, paths[i], 1, L, k, topk_ids=step.topk_ids, topk_logq=step.topk_logq,
+            lse=step.lse, ws=step.ws_topk, stream=s)
+    out = {}
+    for name, fn in calls.items():
+        def run(s, fn=fn):
+            for i, st in enumerate(sets):
+                fn(st, s, i)
+        with torch.cuda.stream(side):
+            run(side)
+        side.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=side):
+            run(side)
+        with torch.cuda.stream(side):
+            for _ in range(3):
+                g.replay()
+            ea = torch.cuda.Event(enable_timing=True)
+            eb = torch.cuda.Event(enable_timing=True)
+            ea.record(side)
+            for _ in range(args.kernel_steps):
+                g.replay()
+            eb.record(side)
+        side.synchronize()
+        out[name] = ea.elapsed_time(eb) * 1e3 / (args.kernel_steps * len(sets))
+        del g
+    del slots
+    torch.cuda.synchronize()
+    if int(step.dev_status.item()) != 0:
+        raise RuntimeError(f"device status after variants: "
+                           f"{P.dev_status_names(int(step.dev_status.item()))}")
+    return out
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -376,6 +453,13 @@ def run_ours(args):
         del g
     torch.cuda.synchronize()
 
+    # ---- the paper's variants of the same calls, timed the same way: beam search
+    # (W = 10), Alg. 2 as printed, a per-row lambda, top-k with entropy-adaptive
+    # lambda, and the self-speculative top-k over the accepted node's mask slots
+    variant_us = None
+    if not args.no_variants:
+        variant_us = time_variants(args, P, w, step, sets, side, ngram)
+
     # ---- end to end through the public API with host buffers
     host = []
     for st in sets:
@@ -493,6 +577,7 @@ def run_ours(args):
             "roofline": roof,
             "topk_hbm_frac": topk_frac,
             "call_us": us,
+            "variant_us": variant_us,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "steps/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h,

@@ -144,6 +144,7 @@ __device__ __forceinline__ void merge_mst(float& m2, float& s, float& t, float n
 struct Plan {
   int rows, parts, vpt, vmax;  // vpt: vectors per thread; vmax: the kernel's register bound
   int epv;                     // elements per 16-byte vector
+  bool stream;                 // streaming kernel (then vpt = vectors per span)
 };
 
 struct Args {
@@ -205,14 +206,89 @@ struct Smem {
 };
 
 // Keys e[0..M) (unique, nonzero) -> their descending top-k in out[0..min(M, k)).
-// Block-wide: every thread takes keys tid, tid + kThreads, ...; no barrier inside.
+// NT threads: every thread takes keys tid, tid + NT, ...; no barrier inside.
+template <int NT = kThreads>
 __device__ __forceinline__ void rank_keys(const unsigned long long* e, int M, int k,
                                           unsigned long long* out, int tid) {
-  for (int i = tid; i < M; i += kThreads) {
+  for (int i = tid; i < M; i += NT) {
     const unsigned long long ki = e[i];
     int r = 0;
     for (int j = 0; j < M; ++j) r += e[j] > ki;
     if (r < k) out[r] = ki;
+  }
+}
+
+// Combine the spans of a row in the leader CTA of its cluster (keys, (max, sum) and
+// the entropy sums), then write the row.  Every thread of the CTA calls this; the
+// first NT take part in ranking; warp 0 holds the CTA's (m, s, t) on entry.
+template <bool ENT, int NT, typename SM>
+__device__ __forceinline__ void finish_row(const Args& a, SM& sh, int row, int part, float m_cta,
+                                           float s_cta, float t_cta, int got) {
+  namespace cg = cooperative_groups;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int k = a.k;
+  // ---- combine the spans of the row in the leader CTA
+  float m_row = m_cta, s_row = s_cta, t_row = t_cta;
+  if (a.parts > 1) {
+    cg::cluster_group cluster = cg::this_cluster();
+    SM* leader = cluster.map_shared_rank(&sh, 0);
+    if (tid < k) leader->part[part][tid] = tid < got ? sh.list[tid] : 0ull;
+    if (tid == 0) {
+      leader->part_ms[part] = make_float2(m_cta, s_cta);
+      if constexpr (ENT) leader->part_t[part] = t_cta;
+    }
+    cluster.sync();
+    if (part != 0) return;
+    // the parts' keys: zeros (fewer than k in a span) rank below every real key and
+    // are dropped below
+    const int P = a.parts * k;
+    for (int i = tid; i < P; i += NT) sh.cand[i] = sh.part[i / k][i % k];
+    if (warp == 0) {
+      float mw = lane < a.parts ? sh.part_ms[lane].x : -INFINITY;
+      float sw = lane < a.parts ? sh.part_ms[lane].y : 0.f;
+      float tw = 0.f;
+      if constexpr (ENT) tw = lane < a.parts ? sh.part_t[lane] : 0.f;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const float m_o = __shfl_xor_sync(kFull, mw, off);
+        const float s_o = __shfl_xor_sync(kFull, sw, off);
+        if constexpr (ENT) {
+          const float t_o = __shfl_xor_sync(kFull, tw, off);
+          merge_mst(mw, sw, tw, m_o, s_o, t_o);
+        } else {
+          merge_ms(mw, sw, m_o, s_o);
+        }
+      }
+      m_row = mw;
+      s_row = sw;
+      t_row = tw;
+    }
+    __syncthreads();
+    rank_keys<NT>(sh.cand, P, k, sh.list, tid);
+    __syncthreads();
+  }
+  // ---- write the row (warp 0 holds the row's (max, sum))
+  if (warp == 0) {
+    // natural-log normaliser: lse = (m2 + log2 s) ln 2 = max + ln s; log q = (x - max) - ln s
+    const float mx = m_row * (1.f / kLog2e);
+    const float logs = logf(s_row);
+    if (lane == 0 && !(mx > -INFINITY && mx < INFINITY)) report(a.dev_status, PRESTO_DEV_NONFINITE);
+    if (lane < k) {
+      const unsigned long long key = sh.list[lane];
+      a.topk_ids[static_cast<size_t>(row) * k + lane] = key_id(key);
+      a.topk_logq[static_cast<size_t>(row) * k + lane] = (key_value(key) - mx) - logs;
+    }
+    if (lane == 0 && a.lse) a.lse[row] = mx + logs;
+    if constexpr (ENT) {
+      if (lane == 0) {
+        // H = -Σ q ln q = ln s - ln2 (t / s); q ln q -> 0 where q underflows.  H >= 0
+        // exactly; rounding can take a near-one-hot row a hair below, so clamp (this
+        // also keeps lambda_d >= 0, as the tree build requires)
+        const float H = fmaxf(logs - 0.6931471805599453f * __fdiv_rn(t_row, s_row), 0.f);
+        if (a.entropy) a.entropy[row] = H;
+        if (a.lambda_d) a.lambda_d[row] = __fdiv_rn(__fmul_rn(a.beta, H), __fadd_rn(H, a.C));
+      }
+    }
   }
 }
 
@@ -437,27 +513,329 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
   __syncthreads();
   const int got = M < k ? M : k;
 
-  // ---- combine the spans of the row in the leader CTA
-  float m_row = m_cta, s_row = s_cta, t_row = t_cta;
-  if (a.parts > 1) {
-    cg::cluster_group cluster = cg::this_cluster();
-    Smem* leader = cluster.map_shared_rank(&sh, 0);
-    if (tid < k) leader->part[part][tid] = tid < got ? sh.list[tid] : 0ull;
-    if (tid == 0) {
-      leader->part_ms[part] = make_float2(m_cta, s_cta);
-      if constexpr (ENT) leader->part_t[part] = t_cta;
+  finish_row<ENT, kThreads>(a, sh, row, part, m_cta, s_cta, t_cta, got);
+}
+
+// ---------------------------------------------------------------------------
+// Streaming variant, for problems of more than one wave of the kernel above (many
+// rows): one producer thread keeps a ring of kSStages bulk copies (32 KB each) of
+// the CTA's span in flight while eight consumer warps work on the chunk before, so
+// HBM stays busy for the whole life of the CTA.  A consumer thread takes 8 vectors
+// of each chunk into registers and updates its online (max, Σexp) pair; the
+// candidates are the elements at or above a threshold taken from the first chunk
+// (the k-th largest of its 16 half-warp maxima: at least k elements of the span
+// reach it), kept in a shared buffer that is cut back to the running top-k (and
+// the threshold raised to its k-th key) whenever it passes half full.  A chunk whose
+// candidates overflow the buffer is re-scanned from registers with a raised key
+// threshold, as in the kernel above.
+// ---------------------------------------------------------------------------
+constexpr int kSCons = 256;                 // consumer threads (8 warps)
+constexpr int kSWarps = kSCons / 32;
+constexpr int kSThreads = kSCons + 32;      // + the producer warp
+constexpr int kSVec = 8;                    // 16-byte vectors per consumer thread and chunk
+constexpr int kSChunkVec = kSCons * kSVec;  // 2048 vectors
+constexpr int kSChunkBytes = kSChunkVec * 16;
+constexpr int kSStages = 3;
+
+constexpr size_t kSDynBytes = static_cast<size_t>(kSStages) * kSChunkBytes + 128;
+static_assert(2 * kSWarps >= kMaxK, "theta needs at least k half-warp maxima");
+constexpr int kSCap = 1024;                 // candidate buffer
+constexpr int kSCompact = kSCap / 2;        // cut back above this many
+static_assert(kSCompact % kSCons == 0, "old candidates are re-read in whole rounds");
+
+struct SSmem {
+  uint64_t full[kSStages], empty[kSStages];
+  unsigned long long cand[kSWarps * kMaxK];  // the warps' top-k; the parts' in the leader
+  unsigned long long list[kMaxK];
+  unsigned long long part[kMaxParts][kMaxK];
+  float2 part_ms[kMaxParts];
+  float part_t[kMaxParts];
+  float2 warp_ms[kSWarps];
+  float warp_t[kSWarps];
+  unsigned long long cand2[kSCap];  // the span's candidates
+  float gmax[2 * kSWarps];  // half-warp maxima of the first chunk
+  float theta;              // the first chunk's threshold, for every consumer
+  int cnt[3];               // candidates appended by chunk c, at cnt[c % 3]
+  int fcnt;                 // the same on the overflow path
+  int abort;                // set by any thread whose bounded wait ran out
+  int stop[2];              // the consumers' common copy of abort at chunk c's end
+};
+
+__device__ __forceinline__ void consumers_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kSCons) : "memory");
+}
+
+template <typename T, bool ENT>
+__global__ void __launch_bounds__(kSThreads, 2) topk_stream_kernel(const Args a) {
+  using E = Elem<T>;
+  constexpr int n = E::kPerVec;
+  constexpr int eb = E::kBytes;
+  __shared__ SSmem sh;
+  extern __shared__ unsigned char dyn_raw[];
+  unsigned char* const ring = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(dyn_raw) + 127) & ~static_cast<uintptr_t>(127));
+  pdl_launch_dependents();
+  const int row = blockIdx.x / a.parts;
+  const int part = blockIdx.x % a.parts;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int k = a.k, V = a.V;
+  if (tid == 0) {
+    for (int st = 0; st < kSStages; ++st) {
+      mbar_init(&sh.full[st], 1);
+      mbar_init(&sh.empty[st], kSWarps);
     }
-    cluster.sync();
-    if (part != 0) return;
-    // the parts' keys: zeros (fewer than k in a span) rank below every real key and
-    // are dropped below
-    const int P = a.parts * k;
-    for (int i = tid; i < P; i += kThreads) sh.cand[i] = sh.part[i / k][i % k];
+    for (int i = 0; i < 3; ++i) sh.cnt[i] = 0;
+    sh.abort = 0;
+    sh.theta = -INFINITY;
+    fence_barrier_init();
+  }
+  __syncthreads();
+  pdl_wait();  // the logits (and slot rows' accept results) come from earlier kernels
+  const T* rowp = row_base<T>(a, row, part == 0 && tid == 0);
+  const int mis = static_cast<int>(reinterpret_cast<uintptr_t>(rowp) & 15);
+  const int head = min(V, mis == 0 ? 0 : (16 - mis) / eb);
+  const int nvec = (V - head) / n;
+  const int tail0 = head + nvec * n;
+  const uint4* vecp = reinterpret_cast<const uint4*>(rowp + head);
+  const int v0 = min(nvec, part * a.vpt);  // vpt: vectors per span here
+  const int v1 = min(nvec, v0 + a.vpt);
+  const int nch = (v1 - v0 + kSChunkVec - 1) / kSChunkVec;
+  volatile int* abort = &sh.abort;
+
+  float m_cta = -INFINITY, s_cta = 0.f, t_cta = 0.f;
+  int got = 0;
+  if (warp == kSWarps) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int c = 0;
+      for (; c < nch; ++c) {
+        const int st = c % kSStages;
+        if (c >= kSStages && !mbar_wait(&sh.empty[st], (c / kSStages - 1) & 1, abort)) {
+          *abort = 1;
+          report(a.dev_status, PRESTO_DEV_TIMEOUT);
+          break;
+        }
+        const int vb = v0 + c * kSChunkVec;
+        const int nv = min(kSChunkVec, v1 - vb);
+        mbar_arrive_expect_tx(&sh.full[st], static_cast<uint32_t>(nv) * 16u);
+        bulk_g2s(ring + st * kSChunkBytes, vecp + vb, static_cast<uint32_t>(nv) * 16u,
+                 &sh.full[st]);
+      }
+      // no copy may still be landing when the CTA exits (the consumers have waited
+      // for every one already unless they gave up)
+      for (int c2 = c > kSStages ? c - kSStages : 0; c2 < c; ++c2)
+        mbar_wait(&sh.full[c2 % kSStages], (c2 / kSStages) & 1, nullptr);
+    }
+  } else {
+    // ------------------------------------------------------------ consumers
+    // extra scalar element: threads 0-6 of part 0 take the head, 8-14 of the last
+    // part the tail (each < 8 elements), with the first chunk
+    int xid = -1;
+    if (part == 0 && tid < head) xid = tid;
+    if (part == a.parts - 1 && tid >= 8 && tid - 8 < V - tail0) xid = tail0 + (tid - 8);
+    const float xval0 = xid >= 0 ? E::load(rowp + xid) : -INFINITY;
+    float mt = -INFINITY, st = 0.f, tt = 0.f;  // running max (plain), Σ 2^u, Σ 2^u u
+    float theta = -INFINITY;                   // candidates: value >= theta ...
+    unsigned long long thr = 1ull;             // ... and key >= thr (every real key is >= 1)
+    int base = 0;                              // candidates kept from earlier chunks
+    const int nloop = nch > 0 ? nch : 1;       // one round for the scalars alone
+    for (int c = 0; c < nloop; ++c) {
+      const int sg = c % kSStages;
+      const int vb = v0 + c * kSChunkVec;
+      const int nv = c < nch ? min(kSChunkVec, v1 - vb) : 0;
+      bool ok = true;
+      if (c < nch && !mbar_wait(&sh.full[sg], (c / kSStages) & 1, abort)) {
+        ok = false;
+        *abort = 1;
+        report(a.dev_status, PRESTO_DEV_TIMEOUT);
+      }
+      uint4 d[kSVec];
+      const uint32_t ni = E::kNegInfWord;
+      auto load_chunk = [&]() {
+#pragma unroll
+        for (int i = 0; i < kSVec; ++i) {
+          const int vi = i * kSCons + tid;
+          d[i] = (ok && vi < nv)
+                     ? *reinterpret_cast<const uint4*>(ring + sg * kSChunkBytes + vi * 16)
+                     : make_uint4(ni, ni, ni, ni);
+        }
+      };
+      load_chunk();  // the slot is released once the chunk's candidates are taken
+      const float xval = c == 0 ? xval0 : -INFINITY;
+      const bool xin = c == 0 && xid >= 0;
+
+      // ---- the chunk's maximum and the online (max, Σ 2^u) pair, log2 domain
+      float cm = xval;
+#pragma unroll
+      for (int i = 0; i < kSVec; ++i) cm = fmaxf(cm, E::vmax(d[i]));
+      if (cm > mt) {
+        if (mt != -INFINITY) {
+          const float dl = mt * kLog2e - cm * kLog2e;  // the old reference minus the new
+          const float f = ex2(dl);
+          if constexpr (ENT) tt = f * fmaf(dl, st, tt);
+          st *= f;
+        }
+        mt = cm;
+      }
+      if (mt != -INFINITY) {
+        const float m2 = mt * kLog2e;
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+        if constexpr (!ENT) {
+#pragma unroll
+          for (int i = 0; i < kSVec; ++i)
+#pragma unroll
+            for (int e = 0; e < n; ++e) acc[e & 3] += ex2(fmaf(E::value(d[i], e), kLog2e, -m2));
+          if (xin) acc[0] += ex2(fmaf(xval, kLog2e, -m2));
+        } else {
+          // u clamped at -256: 2^u flushes to 0 there, so -inf adds 0 to both sums
+          float tac[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+          for (int i = 0; i < kSVec; ++i)
+#pragma unroll
+            for (int e = 0; e < n; ++e) {
+              const float u = fmaxf(fmaf(E::value(d[i], e), kLog2e, -m2), -256.f);
+              const float p = ex2(u);
+              acc[e & 3] += p;
+              tac[e & 3] = fmaf(p, u, tac[e & 3]);
+            }
+          if (xin) {
+            const float u = fmaxf(fmaf(xval, kLog2e, -m2), -256.f);
+            const float p = ex2(u);
+            acc[0] += p;
+            tac[0] = fmaf(p, u, tac[0]);
+          }
+          tt += (tac[0] + tac[1]) + (tac[2] + tac[3]);
+        }
+        st += (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      }
+
+      // ---- first chunk: theta = the k-th largest half-warp maximum (CTA-wide, once)
+      if (c == 0) {
+        float hm = cm;
+#pragma unroll
+        for (int off = 8; off > 0; off >>= 1) hm = fmaxf(hm, __shfl_xor_sync(kFull, hm, off));
+        if ((lane & 15) == 0) sh.gmax[warp * 2 + (lane >> 4)] = hm;
+        consumers_sync();
+        if (warp == 0 && lane < 2 * kSWarps) {
+          const float x = sh.gmax[lane];
+          int r = 0;
+#pragma unroll
+          for (int u = 0; u < 2 * kSWarps; ++u) {
+            const float y = sh.gmax[u];
+            r += y > x || (y == x && u < lane);
+          }
+          if (r == k - 1) sh.theta = x;
+        }
+        consumers_sync();
+        theta = sh.theta;
+      }
+
+      // ---- candidates of the chunk (value >= theta, key >= thr), appended one by one
+      // (they are rare) at base + a per-chunk counter.  The counter of chunk c + 2
+      // is cleared right after chunk c's barrier: every thread read it (as chunk
+      // c - 1's) before that barrier, and appends to it only after the next one.
+      auto emit_chunk = [&](unsigned long long thr_k, int* ctr, int at) {
+#pragma unroll
+        for (int i = 0; i < kSVec; ++i) {
+          const int vi = i * kSCons + tid;
+          if (vi < nv && E::vmax(d[i]) >= theta) {
+            const int id0 = head + (vb + vi) * n;
+#pragma unroll
+            for (int e = 0; e < n; ++e) {
+              const float x = E::value(d[i], e);
+              const unsigned long long key = elem_key(x, id0 + e);
+              if (x >= theta && key >= thr_k) {
+                const int j = at + atomicAdd(ctr, 1);
+                if (j < kSCap) sh.cand2[j] = key;
+              }
+            }
+          }
+        }
+        if (xin && xval >= theta) {
+          const unsigned long long key = elem_key(xval, xid);
+          if (key >= thr_k) {
+            const int j = at + atomicAdd(ctr, 1);
+            if (j < kSCap) sh.cand2[j] = key;
+          }
+        }
+      };
+      const int cs = c % 3;
+      emit_chunk(thr, &sh.cnt[cs], base);
+      if (tid == 0) sh.stop[c & 1] = *abort;  // one reading for all consumers
+      consumers_sync();
+      int M = base + sh.cnt[cs];
+      const int stop = sh.stop[c & 1];
+      if (tid == 0) sh.cnt[(c + 2) % 3] = 0;
+      while (M > kSCap) {
+        // overflow: the k-th largest of the buffer's keys bounds the span's top-k
+        // from below; keep the earlier chunks' keys above it and re-scan this one
+        rank_keys<kSCons>(sh.cand2, kSCap, k, sh.list, tid);
+        consumers_sync();
+        thr = sh.list[k - 1];
+        unsigned long long keep[kSCompact / kSCons];
+#pragma unroll
+        for (int j = 0; j < kSCompact / kSCons; ++j) {
+          const int e = j * kSCons + tid;
+          keep[j] = (e < base && sh.cand2[e] >= thr) ? sh.cand2[e] : 0ull;
+        }
+        if (tid == 0) sh.fcnt = 0;
+        consumers_sync();
+#pragma unroll
+        for (int j = 0; j < kSCompact / kSCons; ++j)
+          if (keep[j]) sh.cand2[atomicAdd(&sh.fcnt, 1)] = keep[j];
+        consumers_sync();
+        base = sh.fcnt;
+        consumers_sync();
+        if (tid == 0) sh.fcnt = 0;
+        consumers_sync();
+        load_chunk();  // the chunk again, from its ring slot
+        emit_chunk(thr, &sh.fcnt, base);
+        consumers_sync();
+        M = base + sh.fcnt;
+        consumers_sync();  // every thread has read the counter
+      }
+      __syncwarp();
+      if (c < nch && lane == 0) mbar_arrive(&sh.empty[sg]);  // the slot may be refilled
+      if (M > kSCompact) {
+        // cut back to the running top-k and raise the thresholds to its k-th key
+        rank_keys<kSCons>(sh.cand2, M, k, sh.list, tid);
+        consumers_sync();
+        thr = sh.list[k - 1];
+        if (tid < k) sh.cand2[tid] = sh.list[tid];
+        M = k;
+        consumers_sync();
+      }
+      if (thr > 1ull) theta = fmaxf(theta, key_value(thr));
+      base = M;
+      if (stop) break;
+    }
+    // ---- the span's top-k and its (max, sum) pair
+    rank_keys<kSCons>(sh.cand2, base, k, sh.list, tid);
+    got = base < k ? base : k;
+    const uint32_t wm_o = __reduce_max_sync(kFull, ordered(mt));
+    const float wm = unordered(wm_o);
+    const float wm2 = wm * kLog2e;
+    const float m2 = mt * kLog2e;
+    const float fw = (mt == -INFINITY) ? 0.f : ex2(m2 - wm2);
+    float ws = st * fw;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) ws += __shfl_xor_sync(kFull, ws, off);
+    float wt = 0.f;
+    if constexpr (ENT) {
+      wt = (mt == -INFINITY) ? 0.f : fw * fmaf(m2 - wm2, st, tt);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) wt += __shfl_xor_sync(kFull, wt, off);
+    }
+    if (lane == 0) {
+      sh.warp_ms[warp] = make_float2(wm == -INFINITY ? -INFINITY : wm2, ws);
+      if constexpr (ENT) sh.warp_t[warp] = wt;
+    }
+    consumers_sync();
     if (warp == 0) {
-      float mw = lane < a.parts ? sh.part_ms[lane].x : -INFINITY;
-      float sw = lane < a.parts ? sh.part_ms[lane].y : 0.f;
+      float mw = lane < kSWarps ? sh.warp_ms[lane].x : -INFINITY;
+      float sw = lane < kSWarps ? sh.warp_ms[lane].y : 0.f;
       float tw = 0.f;
-      if constexpr (ENT) tw = lane < a.parts ? sh.part_t[lane] : 0.f;
+      if constexpr (ENT) tw = lane < kSWarps ? sh.warp_t[lane] : 0.f;
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) {
         const float m_o = __shfl_xor_sync(kFull, mw, off);
@@ -469,37 +847,13 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
           merge_ms(mw, sw, m_o, s_o);
         }
       }
-      m_row = mw;
-      s_row = sw;
-      t_row = tw;
-    }
-    __syncthreads();
-    rank_keys(sh.cand, P, k, sh.list, tid);
-    __syncthreads();
-  }
-  // ---- write the row (warp 0 holds the row's (max, sum))
-  if (warp == 0) {
-    // natural-log normaliser: lse = (m2 + log2 s) ln 2 = max + ln s; log q = (x - max) - ln s
-    const float mx = m_row * (1.f / kLog2e);
-    const float logs = logf(s_row);
-    if (lane == 0 && !(mx > -INFINITY && mx < INFINITY)) report(a.dev_status, PRESTO_DEV_NONFINITE);
-    if (lane < k) {
-      const unsigned long long key = sh.list[lane];
-      a.topk_ids[static_cast<size_t>(row) * k + lane] = key_id(key);
-      a.topk_logq[static_cast<size_t>(row) * k + lane] = (key_value(key) - mx) - logs;
-    }
-    if (lane == 0 && a.lse) a.lse[row] = mx + logs;
-    if constexpr (ENT) {
-      if (lane == 0) {
-        // H = -Σ q ln q = ln s - ln2 (t / s); q ln q -> 0 where q underflows.  H >= 0
-        // exactly; rounding can take a near-one-hot row a hair below, so clamp (this
-        // also keeps lambda_d >= 0, as the tree build requires)
-        const float H = fmaxf(logs - 0.6931471805599453f * __fdiv_rn(t_row, s_row), 0.f);
-        if (a.entropy) a.entropy[row] = H;
-        if (a.lambda_d) a.lambda_d[row] = __fdiv_rn(__fmul_rn(a.beta, H), __fadd_rn(H, a.C));
-      }
+      m_cta = mw;
+      s_cta = sw;
+      t_cta = tw;
     }
   }
+  __syncthreads();  // producer and consumers
+  finish_row<ENT, kSCons>(a, sh, row, part, m_cta, s_cta, t_cta, got);
 }
 
 template <typename T, int VMAX, bool ENT>
@@ -578,6 +932,20 @@ Plan make_plan(int B, int L, int V, int elem_bytes, bool ent) {
     }
   }
   p.vmax = p.vpt <= 4 ? 4 : (p.vpt <= 8 ? 8 : 16);
+  p.stream = false;
+  // More than one wave of the register kernel: stream instead, with about one CTA
+  // per SM or more (a row's spans still form one cluster of <= 8 CTAs)
+  const int act = active_clusters(elem_bytes, p.vmax, p.parts, ent);
+  if (act >= 1 && p.rows > act) {
+    const int sms = sm_count();
+    int parts = (sms + p.rows - 1) / p.rows;
+    parts = parts < 1 ? 1 : (parts > kMaxParts ? kMaxParts : parts);
+    const int nv = V / p.epv;  // a row's aligned vectors, up to one
+    while (parts > 1 && (nv + parts - 1) / parts < kSChunkVec / 2) --parts;  // no tiny spans
+    p.stream = true;
+    p.parts = parts;
+    p.vpt = (nv + 1 + parts - 1) / parts;
+  }
   return p;
 }
 
@@ -598,8 +966,33 @@ cudaError_t launch(const Plan& p, const Args& a, cudaStream_t stream) {
   return cudaLaunchKernelEx(&cfg, topk_kernel<T, VMAX, ENT>, a);
 }
 
+template <typename T, bool ENT>
+cudaError_t launch_stream(const Plan& p, const Args& a, cudaStream_t stream) {
+  static const cudaError_t attr = cudaFuncSetAttribute(
+      topk_stream_kernel<T, ENT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      static_cast<int>(kSDynBytes));
+  if (attr != cudaSuccess) return attr;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(p.rows) * p.parts);
+  cfg.blockDim = dim3(kSThreads);
+  cfg.dynamicSmemBytes = kSDynBytes;
+  cfg.stream = stream;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = p.parts;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  at[1] = pdl_attribute();
+  cfg.attrs = at;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, topk_stream_kernel<T, ENT>, a);
+}
+
 template <bool ENT>
 cudaError_t dispatch(int dtype, const Plan& p, const Args& a, cudaStream_t stream) {
+  if (p.stream)
+    return dtype == PRESTO_F32 ? launch_stream<float, ENT>(p, a, stream)
+                               : launch_stream<__nv_bfloat16, ENT>(p, a, stream);
   if (dtype == PRESTO_F32)
     return p.vmax == 4 ? launch<float, 4, ENT>(p, a, stream)
            : p.vmax == 8 ? launch<float, 8, ENT>(p, a, stream)

@@ -150,3 +150,23 @@ def test_bad_accept_path_is_reported_and_reads_the_root():
     root = O.accepted_slot_rows(x.double().numpy(), [0, 0], [[0, -1, -1], [0, -1, -1]], 0, L)
     oids, _, _ = O.topk_logsoftmax(root.reshape(B * L, V), k)
     np.testing.assert_array_equal(ids.cpu().numpy().reshape(B * L, k), oids)
+
+
+def test_slot_topk_many_rows_stream():
+    """B * L rows beyond one wave of the register-resident kernel: slot rows through
+    the streaming kernel."""
+    rng = np.random.default_rng(21)
+    B, N, S, V, L, k = 12, 4, 33, 151936, 32, 6
+    token, parent, n_nodes = _random_tree(rng, B, N, V)
+    depth = _depths(parent, n_nodes)
+    tgt = _planted_targets(rng, token, parent, n_nodes, V)
+    acc, path, bonus = O.accept(token, parent, n_nodes, tgt, int(depth.max()))
+    x = _slot_logits(B, N, S, V, torch.bfloat16, seed=99)
+    ids, logq, lse, ctx2 = P.presto_topk_slots(x.cuda(), to_dev(acc), to_dev(path), 1, L, k,
+                                               node_token=to_dev(token), bonus=to_dev(bonus))
+    torch.cuda.synchronize()
+    oids, ologq, olse, octx = _oracle(x, acc, path, 1, L, k, token, bonus)
+    np.testing.assert_array_equal(ids.cpu().numpy().reshape(B * L, k), oids)
+    assert rel_close(logq.cpu().numpy().reshape(B * L, k), ologq) <= LOGQ_TOL
+    assert rel_close(lse.cpu().numpy().reshape(-1), olse) <= LOGQ_TOL
+    np.testing.assert_array_equal(ctx2.cpu().numpy(), octx)

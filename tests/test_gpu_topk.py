@@ -85,3 +85,30 @@ def test_topk_all_masked_row_reports_nonfinite():
     P.presto_topk(x.cuda(), 2, dev_status=st)
     torch.cuda.synchronize()
     assert int(st.item()) & 0x100
+
+
+@pytest.mark.parametrize("V,dtype,k", [(151936, torch.bfloat16, 8), (1001, torch.bfloat16, 7),
+                                       (4097, torch.float32, 16), (16, torch.float32, 16),
+                                       (70000, torch.float32, 10)])
+def test_topk_many_rows_stream(V, dtype, k):
+    """More rows than one wave of the register-resident kernel holds: the launch
+    streams the rows through a ring of bulk copies instead."""
+    g = torch.Generator().manual_seed(V * 3 + k)
+    x = (torch.randn(8, 60, V, generator=g) * 3).to(dtype)
+    assert _check(x, k) == 0
+
+
+def test_topk_stream_ties_masks_and_adversarial_rows():
+    """Ties on a grid with a masked vocabulary; constant rows (every element a
+    candidate); increasing rows (every chunk beats the threshold of the last):
+    the candidate buffer overflows and the thresholds are raised exactly."""
+    g = torch.Generator().manual_seed(12)
+    x = torch.round(torch.randn(8, 50, 20000, generator=g) * 2) / 2
+    x[:, :, ::3] = -float("inf")
+    assert _check(x.to(torch.bfloat16), 9) == 0
+    assert _check(x, 16) == 0
+    y = torch.randn(8, 50, 70000, generator=g)
+    y[0, :5] = 1.25                                             # constant rows
+    y[1, :5] = torch.linspace(-20, 20, 70000)                   # increasing rows
+    y[2, :5] = torch.linspace(20, -20, 70000)                   # decreasing rows
+    assert _check(y, 12) == 0

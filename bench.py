@@ -248,6 +248,7 @@ def profiled_traffic(kernel):
 
 def time_variants(args, P, w, step, sets, side, ngram):
     import torch
+    import synth
     dev = step.device
     B, L, k, N = w.B, w.L, w.k, w.N
     f32, i32 = torch.float32, torch.int32
@@ -290,7 +291,27 @@ def time_variants(args, P, w, step, sets, side, ngram):
         calls["topk_slots"] = lambda st, s, i: P.presto_topk_slots(
             slots, acc_len, paths[i], 1, L, k, topk_ids=step.topk_ids, topk_logq=step.topk_logq,
             lse=step.lse, ws=step.ws_topk, stream=s)
+    # one whole round at the largest budget the paper sweeps (N = 1024, k = 10)
+    w2 = w.scaled(N=1024, k=10)
+    step2 = P.DraftVerifyStep(w2.B, w2.L, w2.V, w2.k, w2.N, w2.Hq, w2.Hkv, w2.D, w2.T,
+                              logits_dtype=sets[0]["logits"].dtype, b=w2.branching, lam=w2.lam,
+                              ngram=ngram, device=dev)
+    att2 = synth.attention_inputs(w2, device=dev)
+    kv2 = att2.pop("kv_len").to(torch.int32)
+    tgt2 = torch.zeros(w2.B, w2.N, dtype=i32, device=dev)
+    g2 = step2.capture(sets[0]["logits"], sets[0]["ctx"], [att2], kv2, tgt2)
     out = {}
+    for _ in range(3):
+        g2.replay()
+    ea = torch.cuda.Event(enable_timing=True)
+    eb = torch.cuda.Event(enable_timing=True)
+    ea.record()
+    for _ in range(args.kernel_steps):
+        g2.replay()
+    eb.record()
+    torch.cuda.synchronize()
+    out["round_N1024_k10"] = ea.elapsed_time(eb) * 1e3 / args.kernel_steps
+    del g2, step2, att2
     for name, fn in calls.items():
         def run(s, fn=fn):
             for i, st in enumerate(sets):

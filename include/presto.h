@@ -31,9 +31,10 @@
  *     presto_*_workspace() query returns (256-byte aligned).  Their contents on
  *     entry do not matter.  Two calls that run at the same time need two
  *     workspaces.
- *   - Limits: V < 2^18, 1 <= L <= 63, 1 <= b <= k <= 16, 1 <= N <= 256 (these let
- *     the tree-order key pack into 64 bits), D in {64, 128}, Hq % Hkv == 0 with
- *     Hq / Hkv a power of two <= 128.
+ *   - Limits: V < 2^18, 1 <= L <= 63, 1 <= b <= k <= 16, 1 <= N <= 1024 (these let
+ *     the tree-order key pack into 64 bits: S, depth, the token's rank among its
+ *     depth's k candidates, and a 22-bit parent field), D in {64, 128},
+ *     Hq % Hkv == 0 with Hq / Hkv a power of two <= 128.
  *
  * Sizes: B batch (sequences), L drafter block length (tree depth limit), V vocab,
  * k candidates per position, b branching factor, N node budget including the root,
@@ -274,7 +275,7 @@ int presto_score_build_tree(const int32_t* topk_ids, const float* topk_logq, int
  *                 N best nodes of T.  The paper's default (beam width 10, §5.1).
  *               PRESTO_SEARCH_EAGER: Alg. 2 as printed: pop the best frontier node,
  *                 add all its children to T, until |T| >= N; the N best nodes of T.
- *   beam_width  >= 1 (used by PRESTO_SEARCH_BEAM; <= 256).
+ *   beam_width  >= 1 (used by PRESTO_SEARCH_BEAM; <= 1024).
  * "Best" is always the order S desc, depth asc, token asc, parent index asc, and
  * the output is stored in that order (parent index < child index).
  *   ws          presto_build_workspace_ex(B, L, k, N, beam_width) bytes.

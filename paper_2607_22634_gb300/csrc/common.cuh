@@ -22,7 +22,7 @@ namespace presto {
 
 constexpr int kMaxK = 16;
 constexpr int kMaxL = 63;
-constexpr int kMaxN = 256;
+constexpr int kMaxN = 1024;
 constexpr int kMaxV = 1 << 18;
 // A bounded wait gives up after this many SM cycles (about a second).
 constexpr long long kWaitCycles = 2000000000LL;

@@ -37,6 +37,7 @@
 #include <cmath>
 #include <initializer_list>
 #include <mutex>
+#include <type_traits>
 
 #include "common.cuh"
 
@@ -60,6 +61,7 @@ constexpr float kLn2 = 0.6931471805599453f;
 // (128 bf16 packed in pairs, its first 64 columns); O of tile t at 256 + 128t
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kTmemO = 256;
+constexpr int kWidePartialKeys = 1024;  // prefixes shorter than this merge float32 partials
 constexpr int kMaxSplits = 16;  // KV splits of a row block = CTAs of its cluster
 
 struct Args {
@@ -70,7 +72,7 @@ struct Args {
   float scale_log2;
   __nv_bfloat16* out;
   float* lse;
-  uint2* part_o;    // KV splits: O / l of each row as bf16 [CTA][D / 4][2 * kBM] (column quads)
+  float2* part_o;   // KV splits: O / l of each row, float32 [CTA][D / 2][2 * kBM] (column pairs)
   float2* part_ml;  // KV splits: (m, l) per row [CTA][2 * kBM], log2 domain
   int32_t* dev_status;
 };
@@ -203,12 +205,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     kv = kv < 0 ? 0 : a.Tmax;
   }
   const int nn = nn_raw < 0 ? 0 : (nn_raw > a.N ? a.N : nn_raw);
+  // split partials in float32 when the prefix is short: then a row averages few keys,
+  // its values can be as large as single V entries, and the bf16 roundings of P, of a
+  // bf16 partial and of the output could together reach 2e-2 of N(0, 1) values; with
+  // a long prefix bf16 partials (half the merge traffic) lose nothing measurable
+  const bool wide = kv < kWidePartialKeys;
   const int prefix_tiles = (kv + kBN - 1) / kBN;
-  const int per = (prefix_tiles + a.n_splits - 1) / a.n_splits;
-  const int t_begin = min(split * per, prefix_tiles);
-  const int n_prefix = min(prefix_tiles, t_begin + per) - t_begin;
-  const int n_tree = split == a.n_splits - 1 ? (nn + kBN - 1) / kBN : 0;
-  const int nt = n_prefix + n_tree;  // KV tiles of this split (CTA-uniform)
+  // the KV tiles of a row block, prefix tiles then tree tiles, in equal runs over the
+  // splits: this split's local tile j is prefix tile t_begin + j for j < n_prefix,
+  // else tree tile tree0 + (j - n_prefix)
+  const int tree_tiles = (nn + kBN - 1) / kBN;
+  const int total = prefix_tiles + tree_tiles;
+  const int per = (total + a.n_splits - 1) / a.n_splits;
+  const int t_begin = min(split * per, total);
+  const int nt = min(total, t_begin + per) - t_begin;  // KV tiles of this split (CTA-uniform)
+  const int n_prefix = max(0, min(nt, prefix_tiles - t_begin));
+  const int tree0 = t_begin + n_prefix - prefix_tiles;
 
   volatile int* abort = &abort_flag;
   auto fail = [&]() {
@@ -242,7 +254,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         b * a.Hkv + g, &bars.k_full[st]);
           else
             tma_load_3d(dst + p * Ly::kKVPanel, &tm_kt, p * 64, g,
-                        b * a.N + (j - n_prefix) * kBN, &bars.k_full[st]);
+                        b * a.N + (tree0 + j - n_prefix) * kBN, &bars.k_full[st]);
         }
       }
     }
@@ -266,7 +278,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         b * a.Hkv + g, &bars.v_full[st]);
           else
             tma_load_3d(dst + p * Ly::kKVPanel, &tm_vt, p * 64, g,
-                        b * a.N + (j - n_prefix) * kBN, &bars.v_full[st]);
+                        b * a.N + (tree0 + j - n_prefix) * kBN, &bars.v_full[st]);
         }
       }
     }
@@ -374,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           bits[c] = lc >= 32 ? 0xffffffffu : (lc <= 0 ? 0u : (1u << lc) - 1u);
         }
       } else {
-        const int wi = ((j - n_prefix) * kBN) >> 5;
+        const int wi = ((tree0 + j - n_prefix) * kBN) >> 5;
 #pragma unroll
         for (int c = 0; c < 4; ++c) bits[c] = (mrow && wi + c < a.W) ? __ldg(mrow + wi + c) : 0u;
       }
@@ -442,21 +454,38 @@ __global__ void __launch_bounds__(kThreads, 1)
       a.part_ml[prow] = ok ? make_float2(m, l) : make_float2(-INFINITY, 0.f);
       if (ok) {
         tc_fence_after();
-        // the row normalised by its own l, as bf16 (values stay within the range of V),
-        // column-quad-major so that a warp's 32 rows of one quad are 256 contiguous bytes
+        // the row normalised by its own l (values stay within the range of V), laid
+        // out so that a warp's 32 rows of one column group are 256 contiguous bytes:
+        // bf16 column quads, or float32 column pairs when the sequence's prefix is
+        // short (wide_partials)
         const float inv = l > 0.f ? 1.f / l : 0.f;
-        uint2* dst = a.part_o + static_cast<size_t>(blockIdx.x) * (D / 4) * 2 * kBM + t * kBM + r;
+        if (wide) {
+          float2* dst = reinterpret_cast<float2*>(a.part_o) +
+                        static_cast<size_t>(blockIdx.x) * (D / 2) * 2 * kBM + t * kBM + r;
 #pragma unroll 1
-        for (int c = 0; c < D / 32; ++c) {
-          float o[32];
-          tmem_ld32(tO + c * 32, o);
-          tmem_wait_ld();
+          for (int c = 0; c < D / 32; ++c) {
+            float o[32];
+            tmem_ld32(tO + c * 32, o);
+            tmem_wait_ld();
 #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            const __nv_bfloat162 lo = __floats2bfloat162_rn(o[q * 4] * inv, o[q * 4 + 1] * inv);
-            const __nv_bfloat162 hi = __floats2bfloat162_rn(o[q * 4 + 2] * inv, o[q * 4 + 3] * inv);
-            dst[(c * 8 + q) * 2 * kBM] = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
-                                                    *reinterpret_cast<const uint32_t*>(&hi));
+            for (int q = 0; q < 16; ++q)
+              dst[(c * 16 + q) * 2 * kBM] = make_float2(o[q * 2] * inv, o[q * 2 + 1] * inv);
+          }
+        } else {
+          uint2* dst = reinterpret_cast<uint2*>(a.part_o) +
+                       static_cast<size_t>(blockIdx.x) * (D / 4) * 2 * kBM + t * kBM + r;
+#pragma unroll 1
+          for (int c = 0; c < D / 32; ++c) {
+            float o[32];
+            tmem_ld32(tO + c * 32, o);
+            tmem_wait_ld();
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+              const __nv_bfloat162 lo = __floats2bfloat162_rn(o[q * 4] * inv, o[q * 4 + 1] * inv);
+              const __nv_bfloat162 hi = __floats2bfloat162_rn(o[q * 4 + 2] * inv, o[q * 4 + 3] * inv);
+              dst[(c * 8 + q) * 2 * kBM] = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
+                                                      *reinterpret_cast<const uint32_t*>(&hi));
+            }
           }
         }
       }
@@ -534,79 +563,98 @@ __global__ void __launch_bounds__(kThreads, 1)
   const size_t cta0 = static_cast<size_t>(blockIdx.x - split);  // first CTA of the cluster
   const int r0 = split * slice;
   const int nr = max(0, min(R, r0 + slice) - r0);
-  constexpr int kC4 = D / 4;  // 4-column quads per row
-  // One item = one row of the slice x one column quad, rows fastest (coalesced
-  // partial loads).  Each thread's first two items are loaded before the per-row
-  // weights are formed (one thread per row, into shared memory), so the usual case
-  // costs one L2 round trip.
-  const int nitems = nr * kC4;
-  auto load_item = [&](int item, uint2 (&o)[kMaxSplits]) {
-    const int c4 = item / nr, row = r0 + item % nr;
+  // One item = one row of the slice x one column group (a bf16 quad or a float32
+  // pair), rows fastest (coalesced partial loads).  Each thread's first two items are
+  // loaded before the per-row weights are formed (one thread per row, into shared
+  // memory), so the usual case costs one L2 round trip.
+  auto merge = [&](auto wide_tag) {
+    constexpr bool kWide = decltype(wide_tag)::value;
+    using PT = std::conditional_t<kWide, float2, uint2>;
+    constexpr int kCG = kWide ? D / 2 : D / 4;  // column groups per row
+    const PT* part = reinterpret_cast<const PT*>(a.part_o);
+    const int nitems = nr * kCG;
+    auto load_item = [&](int item, PT (&o)[kMaxSplits]) {
+      const int cg = item / nr, row = r0 + item % nr;
 #pragma unroll
-    for (int s = 0; s < kMaxSplits; ++s)
-      o[s] = (item < nitems && s < nsp)
-                 ? __ldcg(a.part_o + ((cta0 + s) * kC4 + c4) * 2 * kBM + row)
-                 : make_uint2(0u, 0u);
-  };
-  uint2 oa[kMaxSplits], ob[kMaxSplits];
-  load_item(tid, oa);
-  load_item(tid + kThreads, ob);
-  if (tid < nr) {
-    // the row's weights over the splits, w_s l_s / L (a split without keys for the row
-    // has m = -inf and weight 0), and its lse
-    const int row = r0 + tid;
-    float2 ml[kMaxSplits];
+      for (int s = 0; s < kMaxSplits; ++s)
+        o[s] = (item < nitems && s < nsp) ? __ldcg(part + ((cta0 + s) * kCG + cg) * 2 * kBM + row)
+                                         : PT{};
+    };
+    PT oa[kMaxSplits], ob[kMaxSplits];
+    load_item(tid, oa);
+    load_item(tid + kThreads, ob);
+    if (tid < nr) {
+      // the row's weights over the splits, w_s l_s / L (a split without keys for the
+      // row has m = -inf and weight 0), and its lse
+      const int row = r0 + tid;
+      float2 ml[kMaxSplits];
 #pragma unroll
-    for (int s = 0; s < kMaxSplits; ++s)
-      ml[s] = s < nsp ? __ldcg(a.part_ml + (cta0 + s) * 2 * kBM + row) : make_float2(-INFINITY, 0.f);
-    float M = -INFINITY;
+      for (int s = 0; s < kMaxSplits; ++s)
+        ml[s] = s < nsp ? __ldcg(a.part_ml + (cta0 + s) * 2 * kBM + row) : make_float2(-INFINITY, 0.f);
+      float M = -INFINITY;
 #pragma unroll
-    for (int s = 0; s < kMaxSplits; ++s) M = fmaxf(M, ml[s].x);
-    float wl[kMaxSplits], L = 0.f;
+      for (int s = 0; s < kMaxSplits; ++s) M = fmaxf(M, ml[s].x);
+      float wl[kMaxSplits], L = 0.f;
 #pragma unroll
-    for (int s = 0; s < kMaxSplits; ++s) {
-      wl[s] = (M == -INFINITY || ml[s].x == -INFINITY) ? 0.f : ex2(ml[s].x - M) * ml[s].y;
-      L += wl[s];
+      for (int s = 0; s < kMaxSplits; ++s) {
+        wl[s] = (M == -INFINITY || ml[s].x == -INFINITY) ? 0.f : ex2(ml[s].x - M) * ml[s].y;
+        L += wl[s];
+      }
+      const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
+      const bool used = node < nn && L > 0.f;
+      const float inv = used ? 1.f / L : 0.f;
+#pragma unroll
+      for (int s = 0; s < kMaxSplits; ++s) mw[tid][s] = wl[s] * inv;
+      mlse[tid] = used ? (M + log2f(L)) * kLn2 : -INFINITY;
     }
-    const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
-    const bool used = node < nn && L > 0.f;
-    const float inv = used ? 1.f / L : 0.f;
+    __syncthreads();
+    auto finish_item = [&](int item, const PT (&o)[kMaxSplits]) {
+      if (item >= nitems) return;
+      const int cg = item / nr, i = item % nr;
+      const int row = r0 + i;
+      const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
+      const int hh = (row % kBM) % a.G;
+      if (node >= a.N) return;
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int s = 0; s < kMaxSplits; ++s) mw[tid][s] = wl[s] * inv;
-    mlse[tid] = used ? (M + log2f(L)) * kLn2 : -INFINITY;
-  }
-  __syncthreads();
-  auto finish_item = [&](int item, const uint2 (&o)[kMaxSplits]) {
-    if (item >= nitems) return;
-    const int c4 = item / nr, i = item % nr;
-    const int row = r0 + i;
-    const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
-    const int hh = (row % kBM) % a.G;
-    if (node >= a.N) return;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-    for (int s = 0; s < kMaxSplits; ++s) {
-      const float w = mw[i][s];  // 0 for absent splits: their (zero) values are unused
-      acc.x += w * __uint_as_float(o[s].x << 16);
-      acc.y += w * __uint_as_float(o[s].x & 0xffff0000u);
-      acc.z += w * __uint_as_float(o[s].y << 16);
-      acc.w += w * __uint_as_float(o[s].y & 0xffff0000u);
+      for (int s = 0; s < kMaxSplits; ++s) {
+        // weight 0: an absent split, or one without keys for this row (an empty
+        // split writes no partial O, so its workspace bytes are whatever is there)
+        const float w = mw[i][s];
+        if (w != 0.f) {
+          if constexpr (kWide) {
+            acc[0] = fmaf(w, o[s].x, acc[0]);
+            acc[1] = fmaf(w, o[s].y, acc[1]);
+          } else {
+            acc[0] = fmaf(w, __uint_as_float(o[s].x << 16), acc[0]);
+            acc[1] = fmaf(w, __uint_as_float(o[s].x & 0xffff0000u), acc[1]);
+            acc[2] = fmaf(w, __uint_as_float(o[s].y << 16), acc[2]);
+            acc[3] = fmaf(w, __uint_as_float(o[s].y & 0xffff0000u), acc[3]);
+          }
+        }
+      }
+      const size_t orow = ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
+      const __nv_bfloat162 lo = __floats2bfloat162_rn(acc[0], acc[1]);
+      if constexpr (kWide) {
+        *reinterpret_cast<__nv_bfloat162*>(a.out + orow + cg * 2) = lo;
+      } else {
+        const __nv_bfloat162 hi = __floats2bfloat162_rn(acc[2], acc[3]);
+        *reinterpret_cast<uint2*>(a.out + orow + cg * 4) =
+            make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+      }
+      if (cg == 0 && a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = mlse[i];
+    };
+    finish_item(tid, oa);
+    finish_item(tid + kThreads, ob);
+    for (int item = tid + 2 * kThreads; item < nitems; item += kThreads) {
+      load_item(item, oa);
+      finish_item(item, oa);
     }
-    const size_t orow = ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
-    const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
-    const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
-    uint2 u2;
-    u2.x = *reinterpret_cast<const uint32_t*>(&lo);
-    u2.y = *reinterpret_cast<const uint32_t*>(&hi);
-    *reinterpret_cast<uint2*>(a.out + orow + c4 * 4) = u2;
-    if (c4 == 0 && a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = mlse[i];
   };
-  finish_item(tid, oa);
-  finish_item(tid + kThreads, ob);
-  for (int item = tid + 2 * kThreads; item < nitems; item += kThreads) {
-    load_item(item, oa);
-    finish_item(item, oa);
-  }
+  if (wide)
+    merge(std::true_type{});
+  else
+    merge(std::false_type{});
 }
 
 // ------------------------------------------------------------------ host side
@@ -651,7 +699,8 @@ Plan make_plan(int B, int N, int Hq, int Hkv, int Tmax, const int* active) {
   p.G = Hq / Hkv;
   p.n_mt = (N * p.G + kBM - 1) / kBM;
   const int prefix_tiles = (Tmax + kBN - 1) / kBN;
-  int max_splits = prefix_tiles / 2 > 1 ? prefix_tiles / 2 : 1;
+  const int tree_tiles = (N + kBN - 1) / kBN;
+  int max_splits = (prefix_tiles + tree_tiles) / 2 > 1 ? (prefix_tiles + tree_tiles) / 2 : 1;
   if (max_splits > kMaxSplits) max_splits = kMaxSplits;
   // Choose row tiles per CTA (2 lets the softmax of one tile hide behind the
   // tensor-core work of the other, and reads K/V once for both) and the split
@@ -668,7 +717,7 @@ Plan make_plan(int B, int N, int Hq, int Hkv, int Tmax, const int* active) {
     for (int s = 1; s <= max_splits; ++s) {
       if (active[s] < 1) continue;
       const double waves = std::ceil(static_cast<double>(units) / active[s]);
-      const double work = (prefix_tiles + 2.0) / s * tile_cost + 3.0;
+      const double work = (prefix_tiles + tree_tiles) / static_cast<double>(s) * tile_cost + 3.0;
       const double cost = waves * work * (1.0 + 0.02 * (s - 1));
       if (cost < best_cost - 1e-9) {
         best_cost = cost;
@@ -742,7 +791,7 @@ extern "C" size_t presto_attn_workspace(int B, int N, int Hq, int Hkv, int D, in
   const int* active = D == 128 ? active_clusters<128>() : active_clusters<64>();
   const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
   if (p.n_splits == 1) return 256;
-  return align_up(p.ctas * 2 * kBM * (static_cast<size_t>(D) * 2 + 8), 256);
+  return align_up(p.ctas * 2 * kBM * (static_cast<size_t>(D) * 4 + 8), 256);
 }
 
 extern "C" int presto_tree_attention(const void* q, const void* k_cache, const void* v_cache,
@@ -766,10 +815,10 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
   const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
   Args a{};
   if (p.n_splits > 1) {
-    const size_t need = p.ctas * 2 * kBM * (static_cast<size_t>(D) * 2 + 8);
+    const size_t need = p.ctas * 2 * kBM * (static_cast<size_t>(D) * 4 + 8);
     if (!ws || reinterpret_cast<uintptr_t>(ws) % 16 || ws_bytes < need) return PRESTO_ERR_WORKSPACE;
-    a.part_o = static_cast<uint2*>(ws);
-    a.part_ml = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.ctas * 2 * kBM * D * 2);
+    a.part_o = static_cast<float2*>(ws);
+    a.part_ml = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.ctas * 2 * kBM * D * 4);
   }
   const uint64_t e = 2;  // bf16 bytes
   CUtensorMap tq, tkc, tvc, tkt, tvt;

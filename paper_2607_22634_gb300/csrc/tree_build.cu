@@ -27,7 +27,6 @@ namespace presto {
 namespace {
 
 constexpr int kThreads = 512;
-constexpr unsigned kFull = 0xffffffffu;
 
 __host__ __device__ inline uint64_t fmix64(uint64_t k) {
   // MurmurHash3 64-bit finaliser (Appleby, public domain).
@@ -88,6 +87,9 @@ struct Args {
   int per_cta;       // contexts each CTA of the cluster scores
   int tables_in_smem;
   unsigned char* g_tables;  // [B][tables_bytes] when the tables do not fit in smem
+  int p2_in_smem;
+  unsigned char* g_p2;      // [B][p2_stride] when the selection scratch does not
+  size_t tables_stride, p2_stride;  // workspace bytes per sequence
   int32_t* node_token;
   int32_t* node_parent;
   int32_t* node_depth;
@@ -107,6 +109,8 @@ __device__ __forceinline__ float unordered(uint32_t o) {
 
 struct Smem {
   int cid[kMaxL][kMaxK];          // candidate tokens of every depth
+  int trk[kMaxL][kMaxK];          // their ranks by token id within the depth
+  int rtok[kMaxL][kMaxK];         // the token of each rank
   float clq[kMaxL][kMaxK];        // their log q
   int ctx0, ctx1;
   float lam[kMaxL];               // lambda of every drafter row
@@ -132,10 +136,17 @@ struct TableLayout {
     bytes = align_up(static_cast<size_t>(nctx) * bf * 8, 16);
   }
 };
-// Child record of candidate j (token t) of depth d+1 under some context, score s.
-__device__ __forceinline__ uint2 kid_record(float s, int d, int t, int j) {
+// Low word of a node key: 63 - depth (6 bits), 15 - the token's rank among its
+// depth's k candidates by token id (4 bits: all nodes of one depth draw their tokens
+// from the same k candidates, so for equal S and depth this orders by token id), then
+// kPMask - the parent field (22 bits).  In a child record the low field holds the
+// candidate index j instead.
+constexpr uint32_t kPMask = 0x3FFFFFu;
+constexpr int kTRankShift = 22;
+// Child record of candidate j (token rank tr) of depth d+1 under some context, score s.
+__device__ __forceinline__ uint2 kid_record(float s, int d, int tr, int j) {
   return make_uint2(__float_as_uint(s), (static_cast<uint32_t>(63 - (d + 1)) << 26) |
-                                            (static_cast<uint32_t>(0x3FFFF - t) << 8) |
+                                            (static_cast<uint32_t>(15 - tr) << kTRankShift) |
                                             static_cast<uint32_t>(j));
 }
 // Flat context id g (over live contexts only) -> (d, ci).
@@ -219,14 +230,14 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
   int16_t* const rkc = reinterpret_cast<int16_t*>(p2 + ly.rkc);
 
   // Child c of a node with score Sp, children context x and candidate index pj, at
-  // depth dc; `pfield` fills the key's last field (255 - the parent's position among
+  // depth dc; `pfield` fills the key's last field (kPMask - the parent's position among
   // the parents of its level).  Returns the key, context and candidate index.
   auto child = [&](uint32_t x, float Sp, int pj, int pfield, int dc, int c, uint64_t& key,
                    uint32_t& xc, int& jc) {
     const uint2 kd = kids[x * nb + c];
     key = (static_cast<uint64_t>(ordered(__fadd_rn(Sp, __uint_as_float(kd.x)))) << 32) |
-          (kd.y & ~0xFFu) | static_cast<uint32_t>(255 - pfield);
-    jc = static_cast<int>(kd.y & 0xFFu);
+          (kd.y & ~kPMask) | (kPMask - static_cast<uint32_t>(pfield));
+    jc = static_cast<int>(kd.y & kPMask);
     xc = dc >= L ? kNoCtx
                  : static_cast<uint32_t>(dc * cs + (!a.use_table ? 0 : (dc == 1 ? jc : pj * k + jc)));
   };
@@ -404,10 +415,10 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
             int lo = 0, hi = X - 1;
             while (lo < hi) {
               const int mid = (lo + hi) >> 1;
-              if ((akey[cur * N + mid] >> 8) > (key >> 8)) lo = mid + 1;
+              if ((akey[cur * N + mid] >> kTRankShift) > (key >> kTRankShift)) lo = mid + 1;
               else hi = mid;
             }
-            for (; lo < X - 1 && (akey[cur * N + lo] >> 8) == (key >> 8); ++lo)
+            for (; lo < X - 1 && (akey[cur * N + lo] >> kTRankShift) == (key >> kTRankShift); ++lo)
               if (apid[cur * N + lo] == i) key = 0ull;
           }
         }
@@ -459,8 +470,10 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
       a.node_score[o] = 0.f;
     } else if (ke != 0ull) {
       const uint32_t lo = static_cast<uint32_t>(ke);
-      a.node_token[o] = 0x3FFFF - static_cast<int>((lo >> 8) & 0x3FFFFu);
-      a.node_depth[o] = 63 - static_cast<int>((lo >> 26) & 63u);
+      const int dd = 63 - static_cast<int>((lo >> 26) & 63u);
+      const int tr = 15 - static_cast<int>((lo >> kTRankShift) & 15u);
+      a.node_token[o] = sm.rtok[dd - 1][tr];
+      a.node_depth[o] = dd;
       a.node_parent[o] = pid;
       a.node_score[o] = unordered(static_cast<uint32_t>(ke >> 32));
     } else {
@@ -481,15 +494,15 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
   const int b = blockIdx.x / kCluster;
-  const int tid = threadIdx.x, lane = tid & 31;
-  const int L = a.L, k = a.k, N = a.N, nb = a.bf, use_table = a.use_table;
+  const int tid = threadIdx.x;
+  const int L = a.L, k = a.k, nb = a.bf, use_table = a.use_table;
   const TableLayout tl(L, k, nb, use_table);
   // leader's tables: in its shared memory (seen through DSMEM) or in the workspace
   unsigned char* tables;
   if (a.tables_in_smem)
     tables = static_cast<unsigned char*>(cluster.map_shared_rank(static_cast<void*>(dyn), 0));
   else
-    tables = a.g_tables + static_cast<size_t>(b) * tl.bytes;
+    tables = a.g_tables + static_cast<size_t>(b) * a.tables_stride;
   uint2* kids = reinterpret_cast<uint2*>(tables);
   // this CTA's staging area: scores and order of its share of the contexts
   const size_t stage_off = a.tables_in_smem ? tl.bytes : 0;
@@ -527,6 +540,20 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
       const int d = i / (k * k), r = i - d * k * k, j1 = r / k, j2 = r - j1 * k;
       if (j1 < j2 && sm.cid[d][j1] == sm.cid[d][j2]) report(a.dev_status, PRESTO_DEV_DUP_SIBLING);
     }
+  // every candidate's rank by (token, index) within its depth (a permutation even
+  // with duplicate tokens), and the inverse map
+  for (int i = tid; i < L * k; i += kThreads) {
+    const int d = i / k, j = i - d * k;
+    const int t = sm.cid[d][j];
+    int r = 0;
+    for (int u = 0; u < k; ++u) {
+      const int tu = sm.cid[d][u];
+      r += tu < t || (tu == t && u < j);
+    }
+    sm.trk[d][j] = r;
+    sm.rtok[d][r] = t;
+  }
+  __syncthreads();
 
   // ---- phase 1: this CTA scores contexts [g0, g1) of the sequence
   const int g0 = rank * a.per_cta;
@@ -625,7 +652,7 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
         const int gl = f / k, j = f - gl * k;
         int d, ci;
         decode_ctx(g0 + gl, k, use_table, d, ci);
-        kids[(d * tl.cs + ci) * nb + j] = kid_record(sc, d, sm.cid[d][j], j);
+        kids[(d * tl.cs + ci) * nb + j] = kid_record(sc, d, sm.trk[d][j], j);
       } else {
         st_s[f] = sc;
       }
@@ -650,7 +677,7 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
         const int ti = sm.cid[d][i];
         rk += (si > sj) || (si == sj && (ti < tj || (ti == tj && i < j)));
       }
-      if (rk < nb) kids[(d * tl.cs + ci) * nb + rk] = kid_record(row[j], d, sm.cid[d][j], j);
+      if (rk < nb) kids[(d * tl.cs + ci) * nb + rk] = kid_record(row[j], d, sm.trk[d][j], j);
     }
   }
   if (!a.tables_in_smem) __threadfence();
@@ -658,8 +685,11 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   if (rank != 0) return;
 
   // ---- phase 2: top-N selection, level by level (leader CTA)
+  unsigned char* const p2 = a.p2_in_smem
+                                ? dyn + stage_off
+                                : a.g_p2 + static_cast<size_t>(b) * a.p2_stride;
   const int n = select_levels(a, sm, a.tables_in_smem ? reinterpret_cast<const uint2*>(dyn) : kids,
-                              dyn + stage_off, tid);
+                              p2, tid);
   if (tid == 0) a.n_nodes[b] = n;
 }
 
@@ -692,26 +722,54 @@ extern "C" int presto_ngram3_insert(const presto_ngram3* t, const uint64_t* keys
 }
 
 namespace {
-// phase-1 staging area of each CTA, reused by the leader for phase 2
-size_t stage_bytes(int per_cta, int k, int N, int bf, int W) {
-  const size_t st = align_up(static_cast<size_t>(per_cta) * k * 4, 16);
-  const size_t p2 = P2Layout(N, bf, W).bytes;
-  return st > p2 ? st : p2;
-}
 int contexts_all(int L, int k, int use_table) {
   if (!use_table) return L;
   return 1 + (L > 1 ? k : 0) + (L > 2 ? (L - 2) * k * k : 0);
+}
+// Where the leader CTA keeps its tables and its selection scratch: in shared memory
+// when they fit (the scratch aliases the phase-1 staging area), otherwise in the
+// workspace, the scratch first to go (it is touched less per byte than the tables).
+struct BuildPlan {
+  bool tables_in_smem, p2_in_smem;
+  size_t smem;       // dynamic shared memory per CTA
+  size_t ws_tables;  // workspace bytes per sequence
+  size_t ws_p2;
+};
+BuildPlan plan_build(int L, int k, int b, int N, int W, int use_table) {
+  const TableLayout tl(L, k, b, use_table);
+  const int per = (contexts_all(L, k, use_table) + kCluster - 1) / kCluster;
+  const size_t st = align_up(static_cast<size_t>(per) * k * 4, 16);
+  const size_t p2 = P2Layout(N, b, W).bytes;
+  const size_t both = st > p2 ? st : p2;
+  BuildPlan pl{true, true, 0, 0, 0};
+  if (tl.bytes + both <= kDynSmemBudget) {
+    pl.smem = tl.bytes + both;
+  } else if (tl.bytes + st <= kDynSmemBudget) {
+    pl.p2_in_smem = false;
+    pl.smem = tl.bytes + st;
+    pl.ws_p2 = align_up(p2, 256);
+  } else if (both <= kDynSmemBudget) {
+    pl.tables_in_smem = false;
+    pl.smem = both;
+    pl.ws_tables = align_up(tl.bytes, 256);
+  } else {
+    pl.tables_in_smem = pl.p2_in_smem = false;
+    pl.smem = st;
+    pl.ws_tables = align_up(tl.bytes, 256);
+    pl.ws_p2 = align_up(p2, 256);
+  }
+  return pl;
 }
 }  // namespace
 
 extern "C" size_t presto_build_workspace_ex(int B, int L, int k, int N, int beam_width) {
   if (B < 1 || L < 1 || k < 1 || N < 1 || beam_width < 1) return 0;
-  // The leader CTA keeps the tables in shared memory when they fit; otherwise they
-  // live here (sized for the prefix-signal case, the larger one).
+  // sized for the larger case (prefix signal, b = k): what any call with these
+  // shapes keeps outside shared memory fits
+  const BuildPlan pl = plan_build(L, k, k, N, beam_width, 1);
+  if (pl.tables_in_smem && pl.p2_in_smem) return 256;
   const TableLayout tl(L, k, k, 1);
-  const int per = (contexts_all(L, k, 1) + kCluster - 1) / kCluster;
-  const size_t smem = tl.bytes + stage_bytes(per, k, N, k, beam_width);
-  return smem <= kDynSmemBudget ? 256 : align_up(B * tl.bytes, 256);
+  return static_cast<size_t>(B) * (align_up(tl.bytes, 256) + align_up(P2Layout(N, k, beam_width).bytes, 256));
 }
 
 extern "C" size_t presto_build_workspace(int B, int L, int k, int N) {
@@ -773,13 +831,16 @@ extern "C" int presto_score_build_tree_ex(const int32_t* topk_ids, const float* 
   a.N = N;
   a.nctx_all = contexts_all(L, k, a.use_table);
   a.per_cta = (a.nctx_all + kCluster - 1) / kCluster;
-  const TableLayout tl(L, k, b, a.use_table);
-  const size_t sb = stage_bytes(a.per_cta, k, N, b, beam_width);
-  a.tables_in_smem = tl.bytes + sb <= kDynSmemBudget;
-  if (!a.tables_in_smem) {
-    if (!ws || reinterpret_cast<uintptr_t>(ws) % 16 || ws_bytes < static_cast<size_t>(B) * tl.bytes)
-      return PRESTO_ERR_WORKSPACE;
+  const BuildPlan pl = plan_build(L, k, b, N, beam_width, a.use_table);
+  a.tables_in_smem = pl.tables_in_smem;
+  a.p2_in_smem = pl.p2_in_smem;
+  const size_t need = static_cast<size_t>(B) * (pl.ws_tables + pl.ws_p2);
+  if (need > 0) {
+    if (!ws || reinterpret_cast<uintptr_t>(ws) % 16 || ws_bytes < need) return PRESTO_ERR_WORKSPACE;
     a.g_tables = static_cast<unsigned char*>(ws);
+    a.g_p2 = static_cast<unsigned char*>(ws) + static_cast<size_t>(B) * pl.ws_tables;
+    a.tables_stride = pl.ws_tables;
+    a.p2_stride = pl.ws_p2;
   }
   a.node_token = node_token;
   a.node_parent = node_parent;
@@ -787,7 +848,7 @@ extern "C" int presto_score_build_tree_ex(const int32_t* topk_ids, const float* 
   a.node_score = node_score;
   a.n_nodes = n_nodes;
   a.dev_status = dev_status;
-  const size_t smem = (a.tables_in_smem ? tl.bytes : 0) + sb;
+  const size_t smem = pl.smem;
   if (smem > kDynSmemBudget) return PRESTO_ERR_UNSUPPORTED;
   static bool attr_set = [] {
     cudaFuncSetAttribute(build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -19,7 +19,7 @@ __global__ void __launch_bounds__(kMaxN) mask_kernel(const int32_t* node_parent,
                                                      int32_t* dev_status) {
   __shared__ int par[kMaxN];
   __shared__ int dep[kMaxN];
-  __shared__ uint32_t rows[kMaxN][kMaxW + 1];
+  extern __shared__ uint32_t rows[];  // [N][W + 1]
   pdl_launch_dependents();
   pdl_wait();  // the tree comes from the previous kernel on the stream
   const int b = blockIdx.x, i = threadIdx.x;
@@ -33,7 +33,7 @@ __global__ void __launch_bounds__(kMaxN) mask_kernel(const int32_t* node_parent,
   if (i < N) {
     par[i] = node_parent[static_cast<size_t>(b) * N + i];
     dep[i] = node_depth[static_cast<size_t>(b) * N + i];
-    for (int w = 0; w < W; ++w) rows[i][w] = 0u;
+    for (int w = 0; w < W; ++w) rows[i * (W + 1) + w] = 0u;
   }
   __syncthreads();
   if (i < n) {
@@ -42,7 +42,7 @@ __global__ void __launch_bounds__(kMaxN) mask_kernel(const int32_t* node_parent,
     // parents strictly decrease, so the walk ends within i steps
     int j = i;
     for (;;) {
-      rows[i][j >> 5] |= 1u << (j & 31);
+      rows[i * (W + 1) + (j >> 5)] |= 1u << (j & 31);
       if (j == 0) break;
       const int p = par[j];
       if (p < 0 || p >= j) {
@@ -56,7 +56,7 @@ __global__ void __launch_bounds__(kMaxN) mask_kernel(const int32_t* node_parent,
   __syncthreads();
   for (int e = i; e < N * W; e += blockDim.x) {
     const int r = e / W, w = e % W;
-    mask[static_cast<size_t>(b) * N * W + e] = rows[r][w];
+    mask[static_cast<size_t>(b) * N * W + e] = rows[r * (W + 1) + w];
   }
   if (i < N) pos_ids[static_cast<size_t>(b) * N + i] = i < n ? kv + dep[i] : -1;
 }
@@ -78,12 +78,11 @@ __global__ void __launch_bounds__(32) accept_kernel(
     n = n < 1 ? 1 : N;
   }
   const size_t base = static_cast<size_t>(b) * N;
-  uint32_t matched[kMaxW];
-#pragma unroll
-  for (int w = 0; w < kMaxW; ++w) {
+  __shared__ uint32_t matched[kMaxW];
+  for (int w = 0; w < W; ++w) {
     const int i = w * 32 + lane;
     bool m = false;
-    if (w < W && i < n) {
+    if (i < n) {
       if (i == 0) {
         m = true;
       } else {
@@ -94,28 +93,27 @@ __global__ void __launch_bounds__(32) accept_kernel(
           report(dev_status, PRESTO_DEV_BAD_PARENT);
       }
     }
-    matched[w] = __ballot_sync(kFull, m);
+    const uint32_t bal = __ballot_sync(kFull, m);
+    if (lane == 0) matched[w] = bal;
   }
+  __syncwarp();
   // deepest accepted node: maximise (depth, -index)
   unsigned bestkey = 0u;
-#pragma unroll
-  for (int w = 0; w < kMaxW; ++w) {
+  for (int w = 0; w < W; ++w) {
     const int i = w * 32 + lane;
-    if (w < W && i < n) {
+    if (i < n) {
       const uint32_t* row = mask + (base + i) * W;
       bool ok = true;
-#pragma unroll
-      for (int u = 0; u < kMaxW; ++u)
-        if (u < W) ok &= (row[u] & ~matched[u]) == 0u;
+      for (int u = 0; u < W; ++u) ok &= (row[u] & ~matched[u]) == 0u;
       if (ok) {
         const int d = node_depth[base + i];
-        const unsigned key = (static_cast<unsigned>(d & 0x3F) << 9) | (511u - i);
+        const unsigned key = (static_cast<unsigned>(d & 0x3F) << 10) | (1023u - i);
         bestkey = bestkey > key ? bestkey : key;
       }
     }
   }
   const unsigned top = __reduce_max_sync(kFull, bestkey);
-  const int best = 511 - static_cast<int>(top & 511u);
+  const int best = 1023 - static_cast<int>(top & 1023u);
   const uint32_t* row = mask + (base + best) * W;
   // path: set bits of the row in increasing index order, written by prefix count
   int written = 0;
@@ -151,8 +149,14 @@ extern "C" int presto_tree_mask(const int32_t* node_parent, const int32_t* node_
   const int W = (N + 31) / 32;
   const int threads = (N + 31) / 32 * 32;
   cudaLaunchConfig_t cfg{};
+  const size_t rows_bytes = static_cast<size_t>(N) * (W + 1) * 4;
+  static const cudaError_t attr_ok = cudaFuncSetAttribute(
+      mask_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      static_cast<int>(static_cast<size_t>(kMaxN) * (kMaxN / 32 + 1) * 4));
+  if (attr_ok != cudaSuccess) return PRESTO_ERR_CUDA;
   cfg.gridDim = dim3(static_cast<unsigned>(B));
   cfg.blockDim = dim3(static_cast<unsigned>(threads));
+  cfg.dynamicSmemBytes = rows_bytes;
   cfg.stream = stream;
   cudaLaunchAttribute attr[1] = {pdl_attribute()};
   cfg.attrs = attr;

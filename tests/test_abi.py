@@ -62,19 +62,19 @@ def test_host_validation_rejects_bad_arguments():
     assert lib.presto_topk(p, 1, 1, 1, 1 << 18, 1 << 18, 4, p, p, N, N, 0, N, N) == -2
     # row stride below V
     assert lib.presto_topk(p, 1, 1, 1, 100, 99, 4, p, p, N, N, 0, N, N) == -1
-    # build: b > k, N > 256, negative lambda
+    # build: b > k, N > 1024, negative lambda
     args = lambda B, L, k, b, lam, Nn: (p, p, B, L, k, b, p, None, ctypes.c_float(lam), Nn,
                                         p, p, p, p, p, N, 0, N, N)
     assert lib.presto_score_build_tree(*args(1, 4, 4, 5, 0.2, 8)) == -1
-    assert lib.presto_score_build_tree(*args(1, 4, 4, 4, 0.2, 257)) == -2
+    assert lib.presto_score_build_tree(*args(1, 4, 4, 4, 0.2, 1025)) == -2
     assert lib.presto_score_build_tree(*args(1, 4, 4, 4, -0.5, 8)) == -1
     assert lib.presto_score_build_tree(*args(1, 64, 4, 4, 0.2, 8)) == -2
-    # build_ex: unknown policy, beam width 0 or above 256
+    # build_ex: unknown policy, beam width 0 or above 1024
     ex = lambda pol, W: (p, p, 1, 4, 4, 4, p, None, ctypes.c_float(0.2), N, pol, W, 8,
                          p, p, p, p, p, N, 0, N, N)
     assert lib.presto_score_build_tree_ex(*ex(3, 1)) == -1
     assert lib.presto_score_build_tree_ex(*ex(1, 0)) == -1
-    assert lib.presto_score_build_tree_ex(*ex(1, 257)) == -2
+    assert lib.presto_score_build_tree_ex(*ex(1, 1025)) == -2
     # topk_entropy: no output, beta or C not positive and finite
     f = ctypes.c_float
     ent = lambda beta, c, H, lam: (p, 1, 1, 1, 10, 10, 2, f(beta), f(c), p, p, N, H, lam, N, 0,
@@ -85,7 +85,7 @@ def test_host_validation_rejects_bad_arguments():
     assert lib.presto_topk_entropy(*ent(1.0, float("inf"), p, p)) == -1
     assert lib.presto_topk_entropy(*ent(1.0, float("nan"), N, p)) == -1
     # mask: N beyond limit
-    assert lib.presto_tree_mask(p, p, p, p, 1, 300, p, p, N, N) == -2
+    assert lib.presto_tree_mask(p, p, p, p, 1, 1100, p, p, N, N) == -2
     # attention: head dim, GQA ratio, misalignment
     att = lambda D, Hq, Hkv, q=p: (q, p, p, p, 64, p, p, p, p, 1, 8, Hq, Hkv, D,
                                    ctypes.c_float(0.1), p, N, N, 0, N, N)

@@ -157,3 +157,14 @@ def test_attention_kv_len_above_capacity_is_reported():
                             dev_status=st)
     torch.cuda.synchronize()
     assert int(st.item()) & 0x4
+
+
+@pytest.mark.parametrize("D,T,kv", [(128, 700, [650]), (128, 4096, [4096]), (64, 300, [0])])
+def test_attention_large_tree_budgets(D, T, kv):
+    """N = 1024 (and 512 for D = 64): up to eight tree-key tiles, dealt out to the KV
+    splits together with the prefix tiles; an empty prefix leaves only tree keys."""
+    B = 1
+    N = 1024 if D == 128 else 512
+    t = _tree(9 + T, B, N, L=16, k=8)
+    inp = _inputs(B, N, 32, 8, D, T, kv, seed=9 + T)
+    _run_and_check(inp, t, N, kv_heads=[0, 5])

@@ -342,6 +342,91 @@ def time_variants(args, P, w, step, sets, side, ngram):
     return out
 
 
+def time_workload_rooflines(args, P, hbm, tc):
+    """Top-k and one attention layer of the larger workloads, each timed the way the
+    per-call numbers are (a graph of launches over inputs that together exceed L2),
+    against the measured peaks: the kernels' rooflines where the work is large enough
+    to approach them."""
+    import numpy as np
+    import torch
+
+    import synth
+    dev = torch.device("cuda", torch.cuda.current_device())
+    out = {}
+    for name in ("self_spec", "batched_ragged", "long_ctx"):
+        w = synth.WORKLOADS[name]
+        x0 = synth.drafter_logits(w).to(dev)
+        nbytes = x0.numel() * x0.element_size()
+        R = max(2, math.ceil(300e6 / nbytes))
+        xs = [x0] + [torch.roll(x0, shifts=i, dims=2) for i in range(1, R)]
+        ids = torch.empty(w.B, w.L, w.k, dtype=torch.int32, device=dev)
+        lq = torch.empty(w.B, w.L, w.k, dtype=torch.float32, device=dev)
+        lse = torch.empty(w.B, w.L, dtype=torch.float32, device=dev)
+        ws_t = torch.empty(max(P.presto_topk_workspace(w.B, w.L, w.V, w.k), 256), dtype=torch.uint8,
+                           device=dev)
+        topk_us = _graph_time(args, lambda s: [P.presto_topk(x, w.k, ids, lq, lse, ws=ws_t, stream=s)
+                                               for x in xs], len(xs))
+        del xs, x0
+        # one attention layer over a full k-ary tree of N nodes (every node used)
+        att = synth.attention_inputs(w, device=dev)
+        kv = att.pop("kv_len").to(torch.int32)
+        par = [-1] + [(i - 1) // w.k for i in range(1, w.N)]
+        dep = [0] * w.N
+        for i in range(1, w.N):
+            dep[i] = dep[par[i]] + 1
+        parent = torch.tensor([par] * w.B, dtype=torch.int32, device=dev)
+        depth = torch.tensor([dep] * w.B, dtype=torch.int32, device=dev)
+        nn = torch.full((w.B,), w.N, dtype=torch.int32, device=dev)
+        mask, _ = P.presto_tree_mask(parent, depth, nn, kv)
+        ws_a = torch.empty(max(P.presto_attn_workspace(w.B, w.N, w.Hq, w.Hkv, w.D, w.T), 256),
+                           dtype=torch.uint8, device=dev)
+        o = torch.empty(w.B, w.N, w.Hq, w.D, dtype=torch.bfloat16, device=dev)
+        ol = torch.empty(w.B, w.N, w.Hq, dtype=torch.float32, device=dev)
+        attn_us = _graph_time(args, lambda s: P.presto_tree_attention(
+            att["q"], att["k_cache"], att["v_cache"], kv, att["k_tree"], att["v_tree"], mask, nn,
+            out=o, lse=ol, ws=ws_a, stream=s), 1)
+        kvh = kv.cpu().numpy()
+        anc = w.B * (sum(dep) + w.N)
+        flops = 4.0 * w.Hq * w.D * (w.N * int(kvh.sum()) + anc)
+        abytes = 2 * w.Hkv * w.D * 2 * (int(kvh.sum()) + w.B * w.N) + 2 * w.B * w.N * w.Hq * w.D * 2
+        out[name] = {
+            "topk_us": topk_us, "topk_gbs": nbytes / (topk_us * 1e-6) / 1e9,
+            "topk_hbm_frac": nbytes / (topk_us * 1e-6) / 1e9 / hbm,
+            "attention_layer_us": attn_us,
+            "attention_tflops": flops / (attn_us * 1e-6) / 1e12,
+            "attention_tensor_frac": flops / (attn_us * 1e-6) / 1e12 / tc,
+            "attention_hbm_frac": abytes / (attn_us * 1e-6) / 1e9 / hbm,
+        }
+        del att, mask
+        torch.cuda.synchronize()
+    return out
+
+
+def _graph_time(args, fn, per_replay):
+    """Per-launch time of fn's launches captured in one CUDA graph (replayed after
+    three warm-up replays), by CUDA events on the launching stream."""
+    import torch
+    side = torch.cuda.Stream()
+    with torch.cuda.stream(side):
+        fn(side)
+    side.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=side):
+        fn(side)
+    reps = max(3, args.kernel_steps // 2)
+    with torch.cuda.stream(side):
+        for _ in range(3):
+            g.replay()
+        ea = torch.cuda.Event(enable_timing=True)
+        eb = torch.cuda.Event(enable_timing=True)
+        ea.record(side)
+        for _ in range(reps):
+            g.replay()
+        eb.record(side)
+    side.synchronize()
+    return ea.elapsed_time(eb) * 1e3 / (reps * per_replay)
+
+
 def run_ours(args):
     import numpy as np
     import torch
@@ -573,6 +658,10 @@ def run_ours(args):
                       f"launches of the call alone (one per input set); per launch")
     topk_frac = topk_bytes / (us["topk"] * 1e-6) / 1e9 / hbm
 
+    by_workload = None
+    if not args.no_variants:
+        by_workload = time_workload_rooflines(args, P, hbm, tc)
+
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         try:
@@ -599,6 +688,7 @@ def run_ours(args):
             "topk_hbm_frac": topk_frac,
             "call_us": us,
             "variant_us": variant_us,
+            "roofline_by_workload": by_workload,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "steps/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h,

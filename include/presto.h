@@ -9,7 +9,8 @@
  *   presto_topk_slots       the same over the mask slots of the accepted node
  *                           (self-speculative rounds)
  *   presto_score_build_tree prefix-aligned scores + best-first tree up to N nodes
- *                           (_ex: beam search / printed Alg. 2, per-position lambda)
+ *                           (_ex: beam search / printed Alg. 2, per-position lambda;
+ *                           _mask: the tree mask and position ids in the same kernel)
  *   presto_tree_mask        ancestor bitmask and position ids of the tree tokens
  *   presto_tree_attention   tree-masked GQA attention against the KV-cache prefix
  *   presto_accept           longest accepted root path under greedy verification
@@ -291,6 +292,26 @@ int presto_score_build_tree_ex(const int32_t* topk_ids, const float* topk_logq, 
                                int32_t* node_depth, float* node_score, int32_t* n_nodes,
                                void* ws, size_t ws_bytes, int32_t* dev_status,
                                presto_stream_t stream);
+
+/*
+ * presto_score_build_tree_mask - presto_score_build_tree_ex that also writes the
+ * tree-attention mask and position ids of the tree it builds, exactly as
+ * presto_tree_mask computes them (§4.3; App. C (I), (IV)), in the same kernel: one
+ * launch and one dependency fewer per round.
+ *
+ *   kv_len, mask, pos_ids  as presto_tree_mask's ([B] int32 in; [B, N, ceil(N/32)]
+ *               uint32 and [B, N] int32 out); non-null together.
+ * Every other argument is as presto_score_build_tree_ex; PRESTO_DEV_BAD_KVLEN when
+ * kv_len[b] < 0.
+ */
+int presto_score_build_tree_mask(const int32_t* topk_ids, const float* topk_logq, int B, int L,
+                                 int k, int b, const int32_t* ctx2, const presto_ngram3* ngram,
+                                 float lambda, const float* lambda_d, int policy, int beam_width,
+                                 int N, int32_t* node_token, int32_t* node_parent,
+                                 int32_t* node_depth, float* node_score, int32_t* n_nodes,
+                                 const int32_t* kv_len, uint32_t* mask, int32_t* pos_ids,
+                                 void* ws, size_t ws_bytes, int32_t* dev_status,
+                                 presto_stream_t stream);
 
 /*
  * presto_tree_mask - tree attention mask and position ids (§4.3 and App. C (I),

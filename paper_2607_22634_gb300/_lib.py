@@ -59,6 +59,9 @@ _SIGS = {
     "presto_score_build_tree_ex": (_I, [_P, _P, _I, _I, _I, _I, _P, ctypes.POINTER(Ngram3),
                                         ctypes.c_float, _P, _I, _I, _I, _P, _P, _P, _P, _P,
                                         _P, ctypes.c_size_t, _P, _P]),
+    "presto_score_build_tree_mask": (_I, [_P, _P, _I, _I, _I, _I, _P, ctypes.POINTER(Ngram3),
+                                          ctypes.c_float, _P, _I, _I, _I, _P, _P, _P, _P, _P,
+                                          _P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "presto_score_build_tree": (_I, [_P, _P, _I, _I, _I, _I, _P, ctypes.POINTER(Ngram3),
                                      ctypes.c_float, _I, _P, _P, _P, _P, _P, _P,
                                      ctypes.c_size_t, _P, _P]),
@@ -318,10 +321,13 @@ def presto_build_workspace(B, L, k, N, beam_width=1) -> int:
 
 def presto_score_build_tree(topk_ids, topk_logq, ctx2, ngram, lam, N, b=None, out=None, ws=None,
                             dev_status=None, stream=None, lambda_d=None,
-                            policy=SEARCH_BEST_FIRST, beam_width=1):
+                            policy=SEARCH_BEST_FIRST, beam_width=1, kv_len=None, mask=None,
+                            pos_ids=None):
     """Returns dict(token, parent, depth, score, n_nodes) of device tensors.
     ``lambda_d`` ([B, L] float32, optional) gives each drafter row its own lambda;
-    ``policy`` is SEARCH_BEST_FIRST, SEARCH_BEAM (with ``beam_width``) or SEARCH_EAGER."""
+    ``policy`` is SEARCH_BEST_FIRST, SEARCH_BEAM (with ``beam_width``) or SEARCH_EAGER.
+    With ``kv_len`` the same kernel also writes the tree mask and position ids
+    (presto_score_build_tree_mask), returned as out["mask"], out["pos_ids"]."""
     B, L, k = topk_ids.shape
     b = k if b is None else b
     dev = topk_ids.device
@@ -338,12 +344,22 @@ def presto_score_build_tree(topk_ids, topk_logq, ctx2, ngram, lam, N, b=None, ou
                "n_nodes": torch.empty(B, dtype=torch.int32, device=dev)}
     ws, nws = _ws(presto_build_workspace(B, L, k, N, beam_width), dev, ws)
     desc = None if ngram is None else ctypes.byref(ngram.desc)
-    st = load().presto_score_build_tree_ex(
+    if kv_len is not None:
+        W = (N + 31) // 32
+        _need(kv_len, torch.int32, (B,), "kv_len")
+        mask = torch.empty(B, N, W, dtype=torch.int32, device=dev) if mask is None else mask
+        pos_ids = torch.empty(B, N, dtype=torch.int32, device=dev) if pos_ids is None else pos_ids
+        _need(mask, torch.int32, (B, N, W), "mask")
+        _need(pos_ids, torch.int32, (B, N), "pos_ids")
+        out["mask"], out["pos_ids"] = mask, pos_ids
+    st = load().presto_score_build_tree_mask(
         _ptr(topk_ids), _ptr(topk_logq), B, L, k, b, _ptr(ctx2), desc, float(lam),
         _ptr(lambda_d), int(policy), int(beam_width), N,
         _ptr(out["token"]), _ptr(out["parent"]), _ptr(out["depth"]), _ptr(out["score"]),
-        _ptr(out["n_nodes"]), _ptr(ws), nws, _ptr(dev_status), _stream(stream))
-    _check(st, "presto_score_build_tree_ex")
+        _ptr(out["n_nodes"]), _ptr(kv_len), _ptr(mask) if kv_len is not None else None,
+        _ptr(pos_ids) if kv_len is not None else None, _ptr(ws), nws, _ptr(dev_status),
+        _stream(stream))
+    _check(st, "presto_score_build_tree_mask")
     return out
 
 

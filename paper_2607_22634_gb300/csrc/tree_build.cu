@@ -95,6 +95,9 @@ struct Args {
   int32_t* node_depth;
   float* node_score;
   int32_t* n_nodes;
+  const int32_t* kv_len;  // fused mask (nullable together with mask, pos_ids)
+  uint32_t* mask;         // [B][N][ceil(N / 32)]
+  int32_t* pos_ids;       // [B][N]
   int32_t* dev_status;
 };
 
@@ -116,6 +119,7 @@ struct Smem {
   float lam[kMaxL];               // lambda of every drafter row
   int nc[2];                      // candidates of a level (phase 2, double-buffered)
   unsigned long long tau;         // the smallest key of a full A (phase 2)
+  int16_t par[kMaxN];             // the output tree's parents (for the fused mask)
 };
 
 // Tables of one sequence, indexed by context c = d * ctx_stride + ci (d = depth of
@@ -463,6 +467,7 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
       ke = akey[(cur ^ 1) * N + i - head];
       pid = apid[(cur ^ 1) * N + i - head];
     }
+    sm.par[i] = static_cast<int16_t>(i == 0 || ke == 0ull ? -1 : pid);
     if (i == 0) {
       a.node_token[o] = sm.ctx1;
       a.node_parent[o] = -1;
@@ -691,6 +696,31 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   const int n = select_levels(a, sm, a.tables_in_smem ? reinterpret_cast<const uint2*>(dyn) : kids,
                               p2, tid);
   if (tid == 0) a.n_nodes[b] = n;
+  if (a.mask) {
+    // the tree-attention mask and position ids (as presto_tree_mask computes them):
+    // word u of row i has bit j set for every ancestor-or-self j of node i in
+    // [32u, 32u + 32); rows of unused nodes are zero, their position -1
+    __syncthreads();
+    const int N = a.N, W = (N + 31) / 32;
+    int kv = a.kv_len[b];
+    if (kv < 0) {
+      if (tid == 0) report(a.dev_status, PRESTO_DEV_BAD_KVLEN);
+    }
+    for (int i = tid; i < N; i += kThreads) {
+      uint32_t* row = a.mask + (static_cast<size_t>(b) * N + i) * W;
+      int depth = -1;
+      for (int u = 0; u < W; ++u) {
+        uint32_t word = 0u;
+        int dd = 0;
+        if (i < n)
+          for (int j = i; j >= 0; j = sm.par[j], ++dd)
+            if ((j >> 5) == u) word |= 1u << (j & 31);
+        row[u] = word;
+        depth = dd - 1;
+      }
+      a.pos_ids[static_cast<size_t>(b) * N + i] = i < n ? kv + depth : -1;
+    }
+  }
 }
 
 }  // namespace
@@ -797,6 +827,20 @@ extern "C" int presto_score_build_tree_ex(const int32_t* topk_ids, const float* 
                                           int32_t* node_depth, float* node_score,
                                           int32_t* n_nodes, void* ws, size_t ws_bytes,
                                           int32_t* dev_status, presto_stream_t stream) {
+  return presto_score_build_tree_mask(topk_ids, topk_logq, B, L, k, b, ctx2, ngram, lambda,
+                                      lambda_d, policy, beam_width, N, node_token, node_parent,
+                                      node_depth, node_score, n_nodes, nullptr, nullptr, nullptr,
+                                      ws, ws_bytes, dev_status, stream);
+}
+
+extern "C" int presto_score_build_tree_mask(
+    const int32_t* topk_ids, const float* topk_logq, int B, int L, int k, int b,
+    const int32_t* ctx2, const presto_ngram3* ngram, float lambda, const float* lambda_d,
+    int policy, int beam_width, int N, int32_t* node_token, int32_t* node_parent,
+    int32_t* node_depth, float* node_score, int32_t* n_nodes, const int32_t* kv_len,
+    uint32_t* mask, int32_t* pos_ids, void* ws, size_t ws_bytes, int32_t* dev_status,
+    presto_stream_t stream) {
+  PRESTO_CHECK_ARG((kv_len && mask && pos_ids) || (!kv_len && !mask && !pos_ids));
   PRESTO_CHECK_ARG(topk_ids && topk_logq && ctx2 && node_token && node_parent && node_depth &&
                    node_score && n_nodes);
   PRESTO_CHECK_ARG(B >= 1 && L >= 1 && k >= 1 && b >= 1 && N >= 1 && b <= k);
@@ -847,6 +891,9 @@ extern "C" int presto_score_build_tree_ex(const int32_t* topk_ids, const float* 
   a.node_depth = node_depth;
   a.node_score = node_score;
   a.n_nodes = n_nodes;
+  a.kv_len = kv_len;
+  a.mask = mask;
+  a.pos_ids = pos_ids;
   a.dev_status = dev_status;
   const size_t smem = pl.smem;
   if (smem > kDynSmemBudget) return PRESTO_ERR_UNSUPPORTED;

@@ -1,12 +1,13 @@
 """One round of the draft-and-verify hot path with resident buffers.
 
 `DraftVerifyStep` owns every intermediate and workspace of a round for fixed
-shapes, so a round is five library calls with no allocation:
+shapes, so a round is a few library calls with no allocation:
 
-    presto_topk -> presto_score_build_tree -> presto_tree_mask
+    presto_topk -> presto_score_build_tree_mask (tree, mask and position ids)
       -> presto_tree_attention (x layers) -> presto_accept
 
-and can be captured once into a CUDA graph and replayed.
+(or, with fuse_mask=False, presto_score_build_tree then presto_tree_mask), and can
+be captured once into a CUDA graph and replayed.
 """
 
 from __future__ import annotations
@@ -18,7 +19,7 @@ from . import _lib as P
 
 class DraftVerifyStep:
     def __init__(self, B, L, V, k, N, Hq, Hkv, D, Tmax, logits_dtype=torch.bfloat16,
-                 b=None, lam=0.2, ngram=None, device="cuda"):
+                 b=None, lam=0.2, ngram=None, device="cuda", fuse_mask=True):
         self.B, self.L, self.V, self.k, self.N = B, L, V, k, N
         self.Hq, self.Hkv, self.D, self.Tmax = Hq, Hkv, D, Tmax
         self.b = k if b is None else b
@@ -50,8 +51,9 @@ class DraftVerifyStep:
         self.ws_attn = torch.empty(max(P.presto_attn_workspace(B, N, Hq, Hkv, D, Tmax), 1),
                                    dtype=u8, device=dev)
         self.graph = None
-
-    CALLS = ("topk", "build", "mask", "attention", "accept")
+        self.fuse_mask = fuse_mask
+        self.CALLS = (("topk", "build", "attention", "accept") if fuse_mask
+                      else ("topk", "build", "mask", "attention", "accept"))
 
     def run(self, logits, ctx2, layers, kv_len, target_token, stream=None, marks=None,
             only=None):
@@ -77,11 +79,12 @@ class DraftVerifyStep:
             mark("topk", 1)
         if on("build"):
             mark("build", 0)
+            fused = dict(kv_len=kv_len, mask=self.mask, pos_ids=self.pos_ids) if self.fuse_mask else {}
             P.presto_score_build_tree(self.topk_ids, self.topk_logq, ctx2, self.ngram, self.lam,
                                       self.N, b=self.b, out=self.tree, ws=self.ws_build,
-                                      dev_status=self.dev_status, stream=s)
+                                      dev_status=self.dev_status, stream=s, **fused)
             mark("build", 1)
-        if on("mask"):
+        if on("mask") and not self.fuse_mask:
             mark("mask", 0)
             P.presto_tree_mask(self.tree["parent"], self.tree["depth"], self.tree["n_nodes"], kv_len,
                                self.mask, self.pos_ids, dev_status=self.dev_status, stream=s)
@@ -102,9 +105,10 @@ class DraftVerifyStep:
             mark("accept", 1)
 
     def kernels_per_round(self, n_layers=1):
-        """Library kernels one round launches: top-k, tree build, mask, accept and
-        one attention kernel per layer (KV splits merge inside the kernel)."""
-        return 4 + n_layers
+        """Library kernels one round launches: top-k, tree build (with the mask when
+        fused, else a mask kernel too), accept and one attention kernel per layer (KV
+        splits merge inside the kernel)."""
+        return (3 if self.fuse_mask else 4) + n_layers
 
     def capture(self, logits, ctx2, layers, kv_len, target_token):
         """Capture one round on these exact input tensors into a CUDA graph."""

@@ -50,6 +50,34 @@ CASES = [
 ]
 
 
+@pytest.mark.parametrize("B,L,k,b,N,lam,with_table,quant", CASES + [(2, 16, 8, None, 1024, 0.2, True, None)])
+def test_fused_mask_matches_oracle(B, L, k, b, N, lam, with_table, quant):
+    """presto_score_build_tree_mask: the tree as presto_score_build_tree builds it,
+    and the mask and position ids of the oracle's tree, bit-exact."""
+    rng = np.random.default_rng(B * 1000 + L * 31 + k * 7 + N)
+    vocab = rng.choice(200000, 300, replace=False)
+    ids, logq = synthetic_candidates(rng, B, L, k, 200000, quant=quant, vocab=vocab)
+    ctx = rng.choice(vocab, size=(B, 2))
+    entries = reachable_table(rng, ids, ctx) if with_table else None
+    table = ngram = None
+    if entries is not None:
+        a, bb, t, lr = entries
+        table = O.make_table(a, bb, t, lr)
+        ngram = P.Ngram3Table.from_entries(a, bb, t, lr, 18, MISS)
+    kv = rng.integers(0, 40000, size=B)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = P.presto_score_build_tree(to_dev(ids), to_dev(logq, torch.float32), to_dev(ctx), ngram,
+                                    lam, N, b=b, dev_status=st, kv_len=to_dev(kv))
+    torch.cuda.synchronize()
+    g = tree_host({k2: v for k2, v in out.items() if k2 not in ("mask", "pos_ids")})
+    o = O.best_first_tree(ids, logq, ctx, table, MISS, lam, b or k, N, "fp32")
+    assert int(st.item()) == 0
+    assert_tree_exact(g, o, B)
+    omask, opos = O.tree_mask(o["parent"], o["depth"], o["n_nodes"], kv, N)
+    np.testing.assert_array_equal(out["mask"].cpu().numpy().view(np.uint32), omask)
+    np.testing.assert_array_equal(out["pos_ids"].cpu().numpy(), opos)
+
+
 @pytest.mark.parametrize("B,L,k,b,N,lam,with_table,quant", CASES)
 def test_build_matches_oracle_fp32(B, L, k, b, N, lam, with_table, quant):
     rng = np.random.default_rng(B * 1000 + L * 31 + k * 7 + N)

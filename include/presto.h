@@ -369,6 +369,9 @@ int presto_tree_attention(const void* q, const void* k_cache, const void* v_cach
  *               j != 0 has node_token[j] == target_token[parent(j)].
  *   accept_path [B, L+1] int32 out: node ids root..deepest, then -1.
  *   bonus       [B] int32 out: target_token of the deepest accepted node.
+ * The ancestor sets are walked through node_parent (the sets the mask rows hold), so
+ * node_depth and mask are not read; they stay in the signature (non-null) so that a
+ * caller can pass the round's arrays unchanged.
  */
 int presto_accept(const int32_t* node_token, const int32_t* node_parent,
                   const int32_t* node_depth, const uint32_t* mask, const int32_t* n_nodes,

@@ -6,7 +6,6 @@
 namespace presto {
 namespace {
 
-constexpr unsigned kFull = 0xffffffffu;
 constexpr int kMaxW = kMaxN / 32;
 
 // One CTA per sequence, one thread per node: walk the parent chain (at most L
@@ -61,76 +60,90 @@ __global__ void __launch_bounds__(kMaxN) mask_kernel(const int32_t* node_parent,
   if (i < N) pos_ids[static_cast<size_t>(b) * N + i] = i < n ? kv + dep[i] : -1;
 }
 
-// One warp per sequence.  match(i) = (i == 0) || token(i) == target(parent(i));
-// node i is accepted iff every node of its mask row matches; the deepest accepted
-// node (unique when siblings carry distinct tokens; lowest index otherwise) ends
-// the path, whose nodes are the set bits of its mask row in index order.
-__global__ void __launch_bounds__(32) accept_kernel(
-    const int32_t* node_token, const int32_t* node_parent, const int32_t* node_depth,
-    const uint32_t* mask, const int32_t* n_nodes, const int32_t* target_token, int N, int W,
-    int L, int32_t* accept_len, int32_t* accept_path, int32_t* bonus, int32_t* dev_status) {
+// One CTA per sequence.  match(i) = (i == 0) || token(i) == target(parent(i)), one
+// bit per node in shared memory; node i is accepted iff every node on its root path
+// matches (its ancestor set, the same set as its mask row), found by walking the
+// parents (at most L steps); the deepest accepted node (unique when siblings carry
+// distinct tokens; lowest index otherwise) ends the accepted path.
+constexpr int kAccThreads = 256;
+__global__ void __launch_bounds__(kAccThreads) accept_kernel(
+    const int32_t* node_token, const int32_t* node_parent, const int32_t* n_nodes,
+    const int32_t* target_token, int N, int L, int32_t* accept_len, int32_t* accept_path,
+    int32_t* bonus, int32_t* dev_status) {
+  __shared__ int16_t par[kMaxN];
+  __shared__ uint32_t matched[kMaxW];
+  __shared__ unsigned wbest[kAccThreads / 32];
   pdl_launch_dependents();
   pdl_wait();  // the tree and the target tokens come from earlier kernels on the stream
-  const int b = blockIdx.x, lane = threadIdx.x;
+  const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   int n = n_nodes[b];
   if (n < 1 || n > N) {
-    if (lane == 0) report(dev_status, PRESTO_DEV_BAD_NNODES);
+    if (tid == 0) report(dev_status, PRESTO_DEV_BAD_NNODES);
     n = n < 1 ? 1 : N;
   }
   const size_t base = static_cast<size_t>(b) * N;
-  __shared__ uint32_t matched[kMaxW];
-  for (int w = 0; w < W; ++w) {
-    const int i = w * 32 + lane;
+  const int nt = blockDim.x;          // a multiple of 32, <= kAccThreads
+  const int Nw = (N + 31) / 32 * 32;  // whole warps: every lane takes part in the ballots
+  for (int i = tid; i < Nw; i += nt) {
     bool m = false;
+    int p = -1;
     if (i < n) {
       if (i == 0) {
         m = true;
       } else {
-        const int p = node_parent[base + i];
-        if (p >= 0 && p < i)
+        p = node_parent[base + i];
+        if (p >= 0 && p < i) {
           m = node_token[base + i] == target_token[base + p];
-        else
+        } else {
           report(dev_status, PRESTO_DEV_BAD_PARENT);
+          p = -1;
+        }
       }
     }
-    const uint32_t bal = __ballot_sync(kFull, m);
-    if (lane == 0) matched[w] = bal;
+    if (i < N) par[i] = static_cast<int16_t>(p);
+    const uint32_t bal = __ballot_sync(0xffffffffu, m);
+    if (lane == 0) matched[i >> 5] = bal;
   }
-  __syncwarp();
-  // deepest accepted node: maximise (depth, -index)
-  unsigned bestkey = 0u;
-  for (int w = 0; w < W; ++w) {
-    const int i = w * 32 + lane;
-    if (i < n) {
-      const uint32_t* row = mask + (base + i) * W;
-      bool ok = true;
-      for (int u = 0; u < W; ++u) ok &= (row[u] & ~matched[u]) == 0u;
-      if (ok) {
-        const int d = node_depth[base + i];
-        const unsigned key = (static_cast<unsigned>(d & 0x3F) << 10) | (1023u - i);
-        bestkey = bestkey > key ? bestkey : key;
+  __syncthreads();
+  // deepest accepted node: maximise (depth, -index); parents precede children, so a
+  // walk ends within i steps
+  unsigned best = 0u;
+  for (int i = tid; i < n; i += nt) {
+    int j = i, d = 0;
+    bool ok = true;
+    while (j > 0) {
+      if (!((matched[j >> 5] >> (j & 31)) & 1u)) {
+        ok = false;
+        break;
       }
+      j = par[j];
+      ++d;
+    }
+    if (ok && j == 0) {
+      const unsigned key = (static_cast<unsigned>(d & 0x3F) << 10) | (1023u - i);
+      best = best > key ? best : key;
     }
   }
-  const unsigned top = __reduce_max_sync(kFull, bestkey);
-  const int best = 1023 - static_cast<int>(top & 1023u);
-  const uint32_t* row = mask + (base + best) * W;
-  // path: set bits of the row in increasing index order, written by prefix count
-  int written = 0;
-  for (int u = 0; u < W; ++u) {
-    const uint32_t bits = row[u];
-    const int i = u * 32 + lane;
-    if ((bits >> lane) & 1u) {
-      const int slot = written + __popc(bits & ((1u << lane) - 1u));
-      if (slot <= L) accept_path[static_cast<size_t>(b) * (L + 1) + slot] = i;
+  best = __reduce_max_sync(0xffffffffu, best);
+  if (lane == 0) wbest[warp] = best;
+  __syncthreads();
+  if (tid == 0) {
+    for (int w = 0; w < nt / 32; ++w) best = best > wbest[w] ? best : wbest[w];
+    const int node = 1023 - static_cast<int>(best & 1023u);
+    int d = static_cast<int>(best >> 10);
+    if (d > L) {
+      report(dev_status, PRESTO_DEV_BAD_PARENT);
+      d = L;
     }
-    written += __popc(bits);
-  }
-  for (int s = written + lane; s <= L; s += 32) accept_path[static_cast<size_t>(b) * (L + 1) + s] = -1;
-  if (lane == 0) {
-    if (written > L + 1) report(dev_status, PRESTO_DEV_BAD_PARENT);
-    accept_len[b] = node_depth[base + best];
-    bonus[b] = target_token[base + best];
+    int32_t* path = accept_path + static_cast<size_t>(b) * (L + 1);
+    for (int s = d + 1; s <= L; ++s) path[s] = -1;
+    int j = node;
+    for (int s = d; s >= 0; --s) {
+      path[s] = j;
+      j = j > 0 ? par[j] : 0;
+    }
+    accept_len[b] = d;
+    bonus[b] = target_token[base + node];
   }
 }
 
@@ -176,17 +189,17 @@ extern "C" int presto_accept(const int32_t* node_token, const int32_t* node_pare
                    accept_len && accept_path && bonus);
   PRESTO_CHECK_ARG(B >= 1 && N >= 1 && L >= 1);
   PRESTO_CHECK_LIMIT(N <= kMaxN && L <= kMaxL);
-  const int W = (N + 31) / 32;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(B));
-  cfg.blockDim = dim3(32);
+  cfg.blockDim = dim3(static_cast<unsigned>(N < kAccThreads ? (N + 31) / 32 * 32 : kAccThreads));
   cfg.stream = stream;
   cudaLaunchAttribute attr[1] = {pdl_attribute()};
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (cudaLaunchKernelEx(&cfg, accept_kernel, node_token, node_parent, node_depth, mask, n_nodes,
-                         target_token, N, W, L, accept_len, accept_path, bonus,
-                         dev_status) != cudaSuccess)
+  (void)mask;      // the ancestor sets are read from node_parent (the mask rows' sets)
+  (void)node_depth;
+  if (cudaLaunchKernelEx(&cfg, accept_kernel, node_token, node_parent, n_nodes, target_token, N,
+                         L, accept_len, accept_path, bonus, dev_status) != cudaSuccess)
     return PRESTO_ERR_CUDA;
   return launch_status();
 }

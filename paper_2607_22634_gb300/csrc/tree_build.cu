@@ -178,11 +178,14 @@ constexpr int kCluster = 8;
 // set C of a level are double-buffered.  Per entry: key, the index of its own children's
 // context (kNoCtx at depth L), its candidate index j, and its parent's node index.
 struct P2Layout {
-  size_t akey, axc, apid, aj, ckey, cxc, cpid, cj, rk, rkc, bytes;
+  size_t akey, axc, apid, aj, ckey, cxc, cpid, cj, rk, rkc, skey, sidx, bytes;
   int nc;  // capacity of one candidate buffer: every child of max(N, W) parents
+  int np;  // the sort buffer: the power of two >= nc
   __host__ __device__ P2Layout(int N, int bf, int W) {
     const size_t na = N;
     nc = (N > W ? N : W) * bf;
+    np = 1;
+    while (np < nc) np <<= 1;
     size_t o = 0;
     akey = o;  o += 2 * na * 8;
     ckey = o;  o += 2 * static_cast<size_t>(nc) * 8;
@@ -193,11 +196,14 @@ struct P2Layout {
     rk = o;    o += align_up((na + nc) * 2, 4);
     rkc = o;   o += align_up(static_cast<size_t>(nc) * 2, 4);
     aj = o;    o += align_up(2 * na, 4);
-    cj = o;    o += align_up(2 * static_cast<size_t>(nc), 4);
+    cj = o;    o += align_up(2 * static_cast<size_t>(nc), 8);
+    skey = o;  o += static_cast<size_t>(np) * 8;
+    sidx = o;  o += static_cast<size_t>(np) * 2;
     bytes = align_up(o, 16);
   }
 };
 constexpr uint32_t kNoCtx = 0xFFFFFFFFu;
+constexpr int kSortMin = 256;  // candidates of a level above which they are sorted first
 
 // Top-N selection of the candidate tree, level by level (leader CTA, all threads).
 //
@@ -232,6 +238,8 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
   uint8_t* const cj = p2 + ly.cj;
   int16_t* const rk = reinterpret_cast<int16_t*>(p2 + ly.rk);
   int16_t* const rkc = reinterpret_cast<int16_t*>(p2 + ly.rkc);
+  uint64_t* const skey = reinterpret_cast<uint64_t*>(p2 + ly.skey);
+  int16_t* const sidx = reinterpret_cast<int16_t*>(p2 + ly.sidx);
 
   // Child c of a node with score Sp, children context x and candidate index pj, at
   // depth dc; `pfield` fills the key's last field (kPMask - the parent's position among
@@ -274,31 +282,87 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
     // a candidate among the candidates alone (beam search keeps the W best)
     const uint64_t* C = ckey + cc * NC;
     const int ne = na + m;
-    for (int e = tid; e < ne; e += kThreads) {
-      int r;
-      if (e < na) {
-        const uint64_t ke = akey[cur * N + e];
-        r = e;
-        for (int i = 0; i < m; ++i) r += C[i] > ke;
-      } else {
-        const int ci = e - na;
-        const uint64_t ke = C[ci];
-        int lo = 0, hi = na;  // A entries with key >= ke
-        while (lo < hi) {
-          const int mid = (lo + hi) >> 1;
-          if (akey[cur * N + mid] >= ke) lo = mid + 1;
-          else hi = mid;
-        }
-        int rc = 0;
-        for (int i = 0; i < m; ++i) {
-          const uint64_t ki = C[i];
-          rc += ki > ke || (ki == ke && i < ci);
-        }
-        rkc[ci] = static_cast<int16_t>(rc);
-        r = lo + rc;
+    if (m > kSortMin) {
+      // many candidates: sort them once (bitonic, descending; keys are unique and
+      // nonzero, zeros pad to a power of two) and take every rank by binary search
+      int P = 1;
+      while (P < m) P <<= 1;
+      for (int i = tid; i < P; i += kThreads) {
+        skey[i] = i < m ? C[i] : 0ull;
+        sidx[i] = static_cast<int16_t>(i);
       }
-      rk[e] = static_cast<int16_t>(r < cap ? r : cap);
-      if (r == cap - 1) sm.tau = e < na ? akey[cur * N + e] : C[e - na];  // the new A's last key
+      __syncthreads();
+      for (int size = 2; size <= P; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+          for (int t = tid; t < P / 2; t += kThreads) {
+            const int i = 2 * t - (t & (stride - 1)), l = i + stride;
+            const uint64_t ki = skey[i], kl = skey[l];
+            const bool desc = (i & size) == 0;  // this block's direction
+            if (desc ? ki < kl : ki > kl) {
+              skey[i] = kl;
+              skey[l] = ki;
+              const int16_t x = sidx[i];
+              sidx[i] = sidx[l];
+              sidx[l] = x;
+            }
+          }
+          __syncthreads();
+        }
+      }
+      for (int q = tid; q < m; q += kThreads) rkc[sidx[q]] = static_cast<int16_t>(q);
+      __syncthreads();
+      for (int e = tid; e < ne; e += kThreads) {
+        int r;
+        if (e < na) {
+          const uint64_t ke = akey[cur * N + e];
+          int lo = 0, hi = m;  // sorted candidates with key > ke
+          while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (skey[mid] > ke) lo = mid + 1;
+            else hi = mid;
+          }
+          r = e + lo;
+        } else {
+          const int ci = e - na;
+          const uint64_t ke = C[ci];
+          int lo = 0, hi = na;  // A entries with key >= ke
+          while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (akey[cur * N + mid] >= ke) lo = mid + 1;
+            else hi = mid;
+          }
+          r = lo + rkc[ci];
+        }
+        rk[e] = static_cast<int16_t>(r < cap ? r : cap);
+        if (r == cap - 1) sm.tau = e < na ? akey[cur * N + e] : C[e - na];  // the new A's last key
+      }
+    } else {
+      for (int e = tid; e < ne; e += kThreads) {
+        int r;
+        if (e < na) {
+          const uint64_t ke = akey[cur * N + e];
+          r = e;
+          for (int i = 0; i < m; ++i) r += C[i] > ke;
+        } else {
+          const int ci = e - na;
+          const uint64_t ke = C[ci];
+          int lo = 0, hi = na;  // A entries with key >= ke
+          while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (akey[cur * N + mid] >= ke) lo = mid + 1;
+            else hi = mid;
+          }
+          int rc = 0;
+          for (int i = 0; i < m; ++i) {
+            const uint64_t ki = C[i];
+            rc += ki > ke || (ki == ke && i < ci);
+          }
+          rkc[ci] = static_cast<int16_t>(rc);
+          r = lo + rc;
+        }
+        rk[e] = static_cast<int16_t>(r < cap ? r : cap);
+        if (r == cap - 1) sm.tau = e < na ? akey[cur * N + e] : C[e - na];  // the new A's last key
+      }
     }
     if (tid == 0) sm.nc[cc ^ 1] = 0;  // the next level's counter (last read a level ago)
     __syncthreads();
@@ -758,7 +822,8 @@ int contexts_all(int L, int k, int use_table) {
 }
 // Where the leader CTA keeps its tables and its selection scratch: in shared memory
 // when they fit (the scratch aliases the phase-1 staging area), otherwise in the
-// workspace, the scratch first to go (it is touched less per byte than the tables).
+// workspace, the tables first to go (the selection scans its scratch over and over;
+// a table record is read once per child generated).
 struct BuildPlan {
   bool tables_in_smem, p2_in_smem;
   size_t smem;       // dynamic shared memory per CTA
@@ -774,14 +839,14 @@ BuildPlan plan_build(int L, int k, int b, int N, int W, int use_table) {
   BuildPlan pl{true, true, 0, 0, 0};
   if (tl.bytes + both <= kDynSmemBudget) {
     pl.smem = tl.bytes + both;
-  } else if (tl.bytes + st <= kDynSmemBudget) {
-    pl.p2_in_smem = false;
-    pl.smem = tl.bytes + st;
-    pl.ws_p2 = align_up(p2, 256);
   } else if (both <= kDynSmemBudget) {
     pl.tables_in_smem = false;
     pl.smem = both;
     pl.ws_tables = align_up(tl.bytes, 256);
+  } else if (tl.bytes + st <= kDynSmemBudget) {
+    pl.p2_in_smem = false;
+    pl.smem = tl.bytes + st;
+    pl.ws_p2 = align_up(p2, 256);
   } else {
     pl.tables_in_smem = pl.p2_in_smem = false;
     pl.smem = st;

@@ -342,6 +342,24 @@ def time_variants(args, P, w, step, sets, side, ngram):
     return out
 
 
+def max_over_ranks(x, device=None):
+    """The largest of every rank's x (the job's time is its slowest replica's); x
+    itself on a single process."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world, steps_per_rank, seconds):
+    """Whole-job rounds per second: every rank ran steps_per_rank rounds (replicas,
+    weak scaling) within the slowest rank's seconds."""
+    return world * steps_per_rank / seconds
+
+
 def time_workload_rooflines(args, P, hbm, tc):
     """Top-k and one attention layer of the larger workloads, each timed the way the
     per-call numbers are (a graph of launches over inputs that together exceed L2),
@@ -519,13 +537,9 @@ def run_ours(args):
         t_wall1 = time.time()
     if world > 1:
         dist.barrier()
-    ms = e0.elapsed_time(e1)
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(e0.elapsed_time(e1), dev)
     clocks = clk.summary(t_wall0, t_wall1)
-    value = world * args.steps / (ms / 1e3)
+    value = job_throughput(world, args.steps, ms / 1e3)
 
     # ---- per-call durations: each call alone, captured n_sets times in a row
     # (rotating over the input sets, so the big inputs come from HBM) into a CUDA
@@ -602,12 +616,8 @@ def run_ours(args):
     t0 = time.perf_counter()
     for i in range(n_e2e):
         e2e_step(i)
-    e2e_s = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([e2e_s], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
-    e2e_value = world * n_e2e / e2e_s
+    e2e_s = max_over_ranks(time.perf_counter() - t0, dev)
+    e2e_value = job_throughput(world, n_e2e, e2e_s)
 
     # ---- roofline of the dominant call
     peaks, peak_src = load_peaks()

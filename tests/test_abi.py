@@ -75,6 +75,11 @@ def test_host_validation_rejects_bad_arguments():
     assert lib.presto_score_build_tree_ex(*ex(3, 1)) == -1
     assert lib.presto_score_build_tree_ex(*ex(1, 0)) == -1
     assert lib.presto_score_build_tree_ex(*ex(1, 1025)) == -2
+    # build_tree_mask: kv_len, mask and pos_ids come together
+    bm = lambda kv, mk, po: (p, p, 1, 4, 4, 4, p, None, ctypes.c_float(0.2), N, 0, 1, 8,
+                             p, p, p, p, p, kv, mk, po, N, 0, N, N)
+    assert lib.presto_score_build_tree_mask(*bm(p, N, p)) == -1
+    assert lib.presto_score_build_tree_mask(*bm(N, p, N)) == -1
     # topk_entropy: no output, beta or C not positive and finite
     f = ctypes.c_float
     ent = lambda beta, c, H, lam: (p, 1, 1, 1, 10, 10, 2, f(beta), f(c), p, p, N, H, lam, N, 0,

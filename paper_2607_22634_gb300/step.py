@@ -41,9 +41,12 @@ class DraftVerifyStep:
         self.pos_ids = torch.empty(B, N, dtype=i32, device=dev)
         self.attn_out = torch.empty(B, N, Hq, D, dtype=bf, device=dev)
         self.attn_lse = torch.empty(B, N, Hq, dtype=f32, device=dev)
-        self.accept_len = torch.empty(B, dtype=i32, device=dev)
-        self.accept_path = torch.empty(B, L + 1, dtype=i32, device=dev)
-        self.bonus = torch.empty(B, dtype=i32, device=dev)
+        # the round's results, contiguous so that one copy brings them to the host:
+        # accept_len [B], accept_path [B, L + 1], bonus [B]
+        self.result = torch.empty(B * (L + 3), dtype=i32, device=dev)
+        self.accept_len = self.result[:B]
+        self.accept_path = self.result[B:B + B * (L + 1)].view(B, L + 1)
+        self.bonus = self.result[B + B * (L + 1):]
         self.dev_status = torch.zeros(1, dtype=i32, device=dev)
         u8 = torch.uint8
         self.ws_topk = torch.empty(max(P.presto_topk_workspace(B, L, V, k), 1), dtype=u8, device=dev)

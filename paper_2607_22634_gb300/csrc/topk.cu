@@ -728,6 +728,27 @@ __global__ void __launch_bounds__(kSThreads, 2) topk_stream_kernel(const Args a)
         }
         consumers_sync();
         theta = sh.theta;
+      } else {
+        // later chunks: every warp publishes its half-warps' running maxima (real
+        // elements, so the k-th largest of the 16 published values still has k
+        // elements at or above it) and raises its own threshold to that k-th largest,
+        // with no barrier: a value another warp has not yet raised is only a looser
+        // bound
+        volatile float* gm = sh.gmax;
+        float hm = mt;
+#pragma unroll
+        for (int off = 8; off > 0; off >>= 1) hm = fmaxf(hm, __shfl_xor_sync(kFull, hm, off));
+        if ((lane & 15) == 0) gm[warp * 2 + (lane >> 4)] = hm;
+        __syncwarp();
+        const float x = lane < 2 * kSWarps ? gm[lane] : -INFINITY;
+        int r = 0;
+#pragma unroll
+        for (int u = 0; u < 2 * kSWarps; ++u) {
+          const float y = __shfl_sync(kFull, x, u);
+          r += y > x || (y == x && u < lane);
+        }
+        const unsigned who = __ballot_sync(kFull, lane < 2 * kSWarps && r == k - 1);
+        theta = fmaxf(theta, __shfl_sync(kFull, x, __ffs(who) - 1));
       }
 
       // ---- candidates of the chunk (value >= theta, key >= thr), appended one by one

@@ -420,6 +420,60 @@ def time_workload_rooflines(args, P, hbm, tc):
     return out
 
 
+def time_full_depth(args, P):
+    """The long-context workload's whole round with every one of its 36 attention layers
+    (independent seeded Q/K/V, ~39 GB of KV cache resident): the full-depth
+    tree-verify time per round."""
+    import numpy as np
+    import torch
+
+    import synth
+    w = synth.WORKLOADS["long_ctx"]
+    dev = torch.device("cuda", torch.cuda.current_device())
+    kv_bytes = w.layers * 2 * w.B * w.Hkv * w.T * w.D * 2
+    free, _ = torch.cuda.mem_get_info(dev)
+    if free < kv_bytes * 1.2 + (8 << 30):
+        return {"skipped": f"needs about {kv_bytes * 1.2 / 1e9:.0f} GB of free device memory"}
+    a, b, t, lr = synth.trigram_entries(w)
+    ngram = P.Ngram3Table.from_entries(a, b, t, lr, w.table_log2_cap, w.miss_logrho, device=dev)
+    logits = synth.drafter_logits(w).to(dev)
+    ctx = synth.ctx_tokens(w).to(dev)
+    layers, kv = [], None
+    for j in range(w.layers):
+        att = synth.attention_inputs(w, layer=j, device=dev)
+        kv = att.pop("kv_len").to(torch.int32)
+        layers.append(att)
+    step = P.DraftVerifyStep(w.B, w.L, w.V, w.k, w.N, w.Hq, w.Hkv, w.D, w.T,
+                             logits_dtype=logits.dtype, b=w.branching, lam=w.lam, ngram=ngram,
+                             device=dev)
+    target = torch.zeros(w.B, w.N, dtype=torch.int32, device=dev)
+    g = step.capture(logits, ctx, layers, kv, target)
+    for _ in range(2):
+        g.replay()
+    ea = torch.cuda.Event(enable_timing=True)
+    eb = torch.cuda.Event(enable_timing=True)
+    reps = 5
+    ea.record()
+    for _ in range(reps):
+        g.replay()
+    eb.record()
+    torch.cuda.synchronize()
+    ms = ea.elapsed_time(eb) / reps
+    n_nodes = step.tree["n_nodes"].cpu().numpy()
+    mask = step.mask.cpu().numpy().view(np.uint32)
+    anc = sum(int(np.unpackbits(mask[q, : int(n_nodes[q])].view(np.uint8)).sum())
+              for q in range(w.B))
+    kvh = kv.cpu().numpy()
+    flops = 4.0 * w.Hq * w.D * (sum(int(kvh[q]) * int(n_nodes[q]) for q in range(w.B)) + anc)
+    del layers, step, g
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return {"workload": "long_ctx: B=8 L=16 k=10 N=256 T=32768, 36 attention layers",
+            "ms_per_round": ms, "rounds_per_s": 1e3 / ms, "gpu_launches_per_round": 3 + w.layers,
+            "attention_tflops": flops * w.layers / (ms * 1e-3) / 1e12,
+            "kv_cache_gb": kv_bytes / 1e9}
+
+
 def _graph_time(args, fn, per_replay):
     """Per-launch time of fn's launches captured in one CUDA graph (replayed after
     three warm-up replays), by CUDA events on the launching stream."""
@@ -720,6 +774,7 @@ def run_ours(args):
     by_workload = None
     if not args.no_variants:
         by_workload = time_workload_rooflines(args, P, hbm, tc)
+        by_workload["long_ctx_full_depth"] = time_full_depth(args, P)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -3,7 +3,7 @@
 The computation lives in libpresto.so (hand-written CUDA, C ABI in
 include/presto.h); this package holds its build script, a ctypes binding with the
 same entry-point names, and `DraftVerifyStep`, which keeps one round's buffers
-resident and replays the five calls (optionally as one CUDA graph).
+resident and replays the round's calls (optionally as one CUDA graph).
 """
 
 from ._lib import (  # noqa: F401

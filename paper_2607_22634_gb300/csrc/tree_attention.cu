@@ -23,11 +23,13 @@
 //     softmax with packed fp32x2 arithmetic, P written back over S with tcgen05.st.
 //     The running maximum is only moved (and O rescaled in TMEM) when it grows by
 //     more than 2^8, so most tiles skip the rescale;
-//   * with several KV splits, the splits of one row block form a thread-block
-//     cluster (up to 16 CTAs): each CTA writes its rows' fp32 (m, l) and O / l as
-//     bf16 to the workspace (column-quad-major, coalesced), the cluster synchronises
-//     (release / acquire), and each CTA merges a slice of the rows over the splits
-//     with log-sum-exp weights, all loads of a row issued together.
+//   * with several KV splits (a row block's prefix and tree-key tiles dealt out in
+//     equal runs), the splits of one row block form a thread-block cluster (up to 16
+//     CTAs): each CTA writes its rows' fp32 (m, l) and O / l to the workspace (bf16
+//     column quads, or float32 column pairs when the prefix is short; coalesced
+//     either way), the cluster synchronises (release / acquire), and each CTA
+//     merges a slice of the rows over the splits with log-sum-exp weights, all loads
+//     of a row issued together.
 // Every wait is bounded; on time-out the CTA records PRESTO_DEV_TIMEOUT and unwinds.
 #include <cuda_bf16.h>
 
@@ -787,7 +789,7 @@ using namespace presto;
 extern "C" size_t presto_attn_workspace(int B, int N, int Hq, int Hkv, int D, int Tmax) {
   if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || Tmax < 1 || (D != 64 && D != 128))
     return 0;
-  // KV splits leave bf16 partial rows and fp32 (m, l) for the in-kernel merge
+  // KV splits leave partial rows (float32 at most) and fp32 (m, l) for the merge
   const int* active = D == 128 ? active_clusters<128>() : active_clusters<64>();
   const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
   if (p.n_splits == 1) return 256;

@@ -64,6 +64,18 @@ struct Elem<float> {
         "f"(__uint_as_float(u.z)));
     return fmaxf(m, __uint_as_float(u.w));
   }
+  // maximum of N vectors (two independent three-input chains)
+  template <int N>
+  __device__ static float max_of(const uint4 (&d)[N]) {
+    float a = fmaxf(__uint_as_float(d[0].x), __uint_as_float(d[0].y));
+    float b = fmaxf(__uint_as_float(d[0].z), __uint_as_float(d[0].w));
+#pragma unroll
+    for (int i = 1; i < N; ++i) {
+      asm("max.f32 %0, %0, %1, %2;" : "+f"(a) : "f"(__uint_as_float(d[i].x)), "f"(__uint_as_float(d[i].y)));
+      asm("max.f32 %0, %0, %1, %2;" : "+f"(b) : "f"(__uint_as_float(d[i].z)), "f"(__uint_as_float(d[i].w)));
+    }
+    return fmaxf(a, b);
+  }
 };
 template <>
 struct Elem<__nv_bfloat16> {
@@ -81,6 +93,22 @@ struct Elem<__nv_bfloat16> {
     asm("max.bf16x2 %0, %1, %2;" : "=r"(b) : "r"(u.z), "r"(u.w));
     asm("max.bf16x2 %0, %0, %1;" : "+r"(a) : "r"(b));
     return fmaxf(__uint_as_float(a << 16), __uint_as_float(a & 0xffff0000u));
+  }
+  // maximum of N vectors: packed maxima along four independent word chains
+  template <int N>
+  __device__ static float max_of(const uint4 (&d)[N]) {
+    uint32_t m0 = d[0].x, m1 = d[0].y, m2 = d[0].z, m3 = d[0].w;
+#pragma unroll
+    for (int i = 1; i < N; ++i) {
+      asm("max.bf16x2 %0, %0, %1;" : "+r"(m0) : "r"(d[i].x));
+      asm("max.bf16x2 %0, %0, %1;" : "+r"(m1) : "r"(d[i].y));
+      asm("max.bf16x2 %0, %0, %1;" : "+r"(m2) : "r"(d[i].z));
+      asm("max.bf16x2 %0, %0, %1;" : "+r"(m3) : "r"(d[i].w));
+    }
+    asm("max.bf16x2 %0, %0, %1;" : "+r"(m0) : "r"(m1));
+    asm("max.bf16x2 %0, %0, %1;" : "+r"(m2) : "r"(m3));
+    asm("max.bf16x2 %0, %0, %1;" : "+r"(m0) : "r"(m2));
+    return fmaxf(__uint_as_float(m0 << 16), __uint_as_float(m0 & 0xffff0000u));
   }
 };
 
@@ -213,8 +241,42 @@ __device__ __forceinline__ void rank_keys(const unsigned long long* e, int M, in
   for (int i = tid; i < M; i += NT) {
     const unsigned long long ki = e[i];
     int r = 0;
-    for (int j = 0; j < M; ++j) r += e[j] > ki;
+    int j = 0;
+    for (; j + 8 <= M; j += 8) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u) r += e[j + u] > ki;
+    }
+    for (; j < M; ++j) r += e[j] > ki;
     if (r < k) out[r] = ki;
+  }
+}
+
+// Warp 0 writes a row: its top-k ids and log q from the k keys in `list`, lse and
+// (ENT) the entropy and lambda_d, from the row's (max log2, Σ 2^u[, Σ 2^u u]).
+template <bool ENT>
+__device__ __forceinline__ void write_row(const Args& a, const unsigned long long* list, int row,
+                                          float m_row, float s_row, float t_row) {
+  const int lane = threadIdx.x & 31;
+  const int k = a.k;
+  // natural-log normaliser: lse = (m2 + log2 s) ln 2 = max + ln s; log q = (x - max) - ln s
+  const float mx = m_row * (1.f / kLog2e);
+  const float logs = logf(s_row);
+  if (lane == 0 && !(mx > -INFINITY && mx < INFINITY)) report(a.dev_status, PRESTO_DEV_NONFINITE);
+  if (lane < k) {
+    const unsigned long long key = list[lane];
+    a.topk_ids[static_cast<size_t>(row) * k + lane] = key_id(key);
+    a.topk_logq[static_cast<size_t>(row) * k + lane] = (key_value(key) - mx) - logs;
+  }
+  if (lane == 0 && a.lse) a.lse[row] = mx + logs;
+  if constexpr (ENT) {
+    if (lane == 0) {
+      // H = -Σ q ln q = ln s - ln2 (t / s); q ln q -> 0 where q underflows.  H >= 0
+      // exactly; rounding can take a near-one-hot row a hair below, so clamp (this
+      // also keeps lambda_d >= 0, as the tree build requires)
+      const float H = fmaxf(logs - 0.6931471805599453f * __fdiv_rn(t_row, s_row), 0.f);
+      if (a.entropy) a.entropy[row] = H;
+      if (a.lambda_d) a.lambda_d[row] = __fdiv_rn(__fmul_rn(a.beta, H), __fadd_rn(H, a.C));
+    }
   }
 }
 
@@ -268,28 +330,7 @@ __device__ __forceinline__ void finish_row(const Args& a, SM& sh, int row, int p
     __syncthreads();
   }
   // ---- write the row (warp 0 holds the row's (max, sum))
-  if (warp == 0) {
-    // natural-log normaliser: lse = (m2 + log2 s) ln 2 = max + ln s; log q = (x - max) - ln s
-    const float mx = m_row * (1.f / kLog2e);
-    const float logs = logf(s_row);
-    if (lane == 0 && !(mx > -INFINITY && mx < INFINITY)) report(a.dev_status, PRESTO_DEV_NONFINITE);
-    if (lane < k) {
-      const unsigned long long key = sh.list[lane];
-      a.topk_ids[static_cast<size_t>(row) * k + lane] = key_id(key);
-      a.topk_logq[static_cast<size_t>(row) * k + lane] = (key_value(key) - mx) - logs;
-    }
-    if (lane == 0 && a.lse) a.lse[row] = mx + logs;
-    if constexpr (ENT) {
-      if (lane == 0) {
-        // H = -Σ q ln q = ln s - ln2 (t / s); q ln q -> 0 where q underflows.  H >= 0
-        // exactly; rounding can take a near-one-hot row a hair below, so clamp (this
-        // also keeps lambda_d >= 0, as the tree build requires)
-        const float H = fmaxf(logs - 0.6931471805599453f * __fdiv_rn(t_row, s_row), 0.f);
-        if (a.entropy) a.entropy[row] = H;
-        if (a.lambda_d) a.lambda_d[row] = __fdiv_rn(__fmul_rn(a.beta, H), __fadd_rn(H, a.C));
-      }
-    }
-  }
+  if (warp == 0) write_row<ENT>(a, sh.list, row, m_row, s_row, t_row);
 }
 
 template <typename T, int VMAX, bool ENT>
@@ -518,76 +559,110 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
 
 // ---------------------------------------------------------------------------
 // Streaming variant, for problems of more than one wave of the kernel above (many
-// rows): one producer thread keeps a ring of kSStages bulk copies (32 KB each) of
-// the CTA's span in flight while eight consumer warps work on the chunk before, so
-// HBM stays busy for the whole life of the CTA.  A consumer thread takes 8 vectors
-// of each chunk into registers and updates its online (max, Σexp) pair; the
-// candidates are the elements at or above a threshold taken from the first chunk
-// (the k-th largest of its 16 half-warp maxima: at least k elements of the span
-// reach it), kept in a shared buffer that is cut back to the running top-k (and
-// the threshold raised to its k-th key) whenever it passes half full.  A chunk whose
-// candidates overflow the buffer is re-scanned from registers with a raised key
-// threshold, as in the kernel above.
+// rows).  The CTA's span is cut into 4 KB chunks that the warps claim one at a time
+// from a counter in shared memory, so a warp whose copies land late takes fewer;
+// each warp's lane 0 keeps kWStages claimed chunks in flight as bulk copies into a
+// ring of the warp's own.  Each chunk's (max, Σ 2^u) pair is summed warp-wide in a
+// fixed order and kept under the chunk's index, and the CTA merges the pairs in chunk
+// order, so the result does not depend on which warp took which chunk.  Every warp
+// keeps its own top-k, sorted across lanes 0..k-1.  A candidate must reach theta: first
+// the k-th largest of all lanes' first-chunk maxima in the CTA (each a real
+// element), then the largest k-th value any warp of the CTA has published (a warp's
+// list holds k elements at or above its k-th value); nothing below theta is in the
+// row's top-k.  A lane whose chunk maximum is below theta costs one compare; a
+// candidate enters the warp's list by a warp-wide sorted insertion.  At the end
+// every warp sends the keys of its list at or above theta, and warp 0 the CTA's
+// (max, sum) pair, straight to the leader CTA of the row's cluster, which merges
+// them after one cluster barrier.
 // ---------------------------------------------------------------------------
-constexpr int kSCons = 256;                 // consumer threads (8 warps)
-constexpr int kSWarps = kSCons / 32;
-constexpr int kSThreads = kSCons + 32;      // + the producer warp
-constexpr int kSVec = 8;                    // 16-byte vectors per consumer thread and chunk
-constexpr int kSChunkVec = kSCons * kSVec;  // 2048 vectors
-constexpr int kSChunkBytes = kSChunkVec * 16;
-constexpr int kSStages = 3;
+constexpr int kWThreads = 256;
+constexpr int kWWarps = kWThreads / 32;
+constexpr int kWVec = 8;                    // 16-byte vectors per lane and chunk
+constexpr int kWChunkVec = 32 * kWVec;      // 256 vectors
+constexpr int kWChunkBytes = kWChunkVec * 16;
+constexpr int kWStages = 3;
+constexpr size_t kWDynBytes = static_cast<size_t>(kWWarps) * kWStages * kWChunkBytes + 128;
+constexpr int kWCtasPerSm = 2;  // ~106 KB of shared memory and <= 128 registers a thread
+constexpr int kWSlots = kMaxParts * kWWarps;  // (part, warp) key lists gathered in the leader
+// chunks of one span at most (a float32 row of fewer than 2^18 elements), plus one
+// pair for the scalar head and tail elements
+constexpr int kWMaxChunks = ((kMaxV / 4) + kWChunkVec - 1) / kWChunkVec + 1;
+static_assert(kWStages == 3, "the claim queue below holds three chunks");
 
-constexpr size_t kSDynBytes = static_cast<size_t>(kSStages) * kSChunkBytes + 128;
-static_assert(2 * kSWarps >= kMaxK, "theta needs at least k half-warp maxima");
-constexpr int kSCap = 1024;                 // candidate buffer
-constexpr int kSCompact = kSCap / 2;        // cut back above this many
-static_assert(kSCompact % kSCons == 0, "old candidates are re-read in whole rounds");
-
-struct SSmem {
-  uint64_t full[kSStages], empty[kSStages];
-  unsigned long long cand[kSWarps * kMaxK];  // the warps' top-k; the parts' in the leader
-  unsigned long long list[kMaxK];
-  unsigned long long part[kMaxParts][kMaxK];
-  float2 part_ms[kMaxParts];
-  float part_t[kMaxParts];
-  float2 warp_ms[kSWarps];
-  float warp_t[kSWarps];
-  unsigned long long cand2[kSCap];  // the span's candidates
-  float gmax[2 * kSWarps];  // half-warp maxima of the first chunk
-  float theta;              // the first chunk's threshold, for every consumer
-  int cnt[3];               // candidates appended by chunk c, at cnt[c % 3]
-  int fcnt;                 // the same on the overflow path
-  int abort;                // set by any thread whose bounded wait ran out
-  int stop[2];              // the consumers' common copy of abort at chunk c's end
+struct WSmem {
+  uint64_t full[kWWarps][kWStages];
+  unsigned long long keys[kWSlots * kMaxK];  // leader: every warp's kept keys (0 = none)
+  unsigned long long list[kMaxK];            // leader: the row's top-k, descending
+  float2 ms[kMaxParts];                      // leader: every part's (max log2, Σ 2^u)
+  float ts[kMaxParts];                       // leader, ENT: every part's Σ 2^u u
+  float2 cms[kWMaxChunks];                   // every chunk's (max log2, Σ 2^u)
+  float cts[kWMaxChunks];                    // ENT: every chunk's Σ 2^u u
+  uint32_t first[kWWarps * kMaxK];           // every warp's k largest first-chunk lane maxima
+  float theta[kWWarps];                      // every warp's published k-th value
+  float theta0;                              // the CTA's first threshold
+  int next;                                  // the next chunk of the span to claim
+  int abort;                                 // set by any warp whose bounded wait ran out
 };
 
-__device__ __forceinline__ void consumers_sync() {
-  asm volatile("bar.sync 1, %0;" ::"n"(kSCons) : "memory");
+// Insert `key` (uniform across the warp, larger than the k-th key) into the warp's
+// descending list lst (lane j < k holds the j-th key, 0 = none); returns the new
+// k-th key.
+__device__ __forceinline__ unsigned long long warp_insert(unsigned long long& lst,
+                                                          unsigned long long key, int k,
+                                                          int lane) {
+  const int pos = __popc(__ballot_sync(kFull, lane < k && lst > key));
+  const unsigned long long up = __shfl_up_sync(kFull, lst, 1);
+  if (lane < k) lst = lane == pos ? key : (lane > pos ? up : lst);
+  return __shfl_sync(kFull, lst, k - 1);
+}
+
+// Merge pairs (m2_j, s_j[, t_j]) (log2-domain maxima, Σ 2^u, Σ 2^u u) held by the
+// lanes of a warp into one, the same in every lane: the maximum by a reduction, then
+// each pair moved to it and summed.  Pairs with m2 = -inf hold nothing.
+template <bool ENT>
+__device__ __forceinline__ void warp_merge_pairs(float& m2, float& s, float& t) {
+  const float M = unordered(__reduce_max_sync(kFull, ordered(m2)));
+  float so = 0.f, to = 0.f;
+  if (m2 != -INFINITY) {
+    const float f = ex2(m2 - M);
+    so = s * f;
+    if constexpr (ENT) to = f * fmaf(m2 - M, s, t);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    so += __shfl_xor_sync(kFull, so, off);
+    if constexpr (ENT) to += __shfl_xor_sync(kFull, to, off);
+  }
+  m2 = M;
+  s = so;
+  t = to;
 }
 
 template <typename T, bool ENT>
-__global__ void __launch_bounds__(kSThreads, 2) topk_stream_kernel(const Args a) {
+__global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a) {
+  namespace cg = cooperative_groups;
   using E = Elem<T>;
   constexpr int n = E::kPerVec;
   constexpr int eb = E::kBytes;
-  __shared__ SSmem sh;
+  __shared__ WSmem sh;
   extern __shared__ unsigned char dyn_raw[];
-  unsigned char* const ring = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(dyn_raw) + 127) & ~static_cast<uintptr_t>(127));
   pdl_launch_dependents();
   const int row = blockIdx.x / a.parts;
   const int part = blockIdx.x % a.parts;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int k = a.k, V = a.V;
-  if (tid == 0) {
-    for (int st = 0; st < kSStages; ++st) {
-      mbar_init(&sh.full[st], 1);
-      mbar_init(&sh.empty[st], kSWarps);
-    }
-    for (int i = 0; i < 3; ++i) sh.cnt[i] = 0;
-    sh.abort = 0;
-    sh.theta = -INFINITY;
+  unsigned char* const ring =
+      reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(dyn_raw) + 127) &
+                                       ~static_cast<uintptr_t>(127)) +
+      warp * kWStages * kWChunkBytes;
+  if (lane == 0) {
+    for (int s = 0; s < kWStages; ++s) mbar_init(&sh.full[warp][s], 1);
+    sh.theta[warp] = -INFINITY;
     fence_barrier_init();
+  }
+  if (tid == 0) {
+    sh.abort = 0;
+    sh.next = 0;
   }
   __syncthreads();
   pdl_wait();  // the logits (and slot rows' accept results) come from earlier kernels
@@ -599,282 +674,312 @@ __global__ void __launch_bounds__(kSThreads, 2) topk_stream_kernel(const Args a)
   const uint4* vecp = reinterpret_cast<const uint4*>(rowp + head);
   const int v0 = min(nvec, part * a.vpt);  // vpt: vectors per span here
   const int v1 = min(nvec, v0 + a.vpt);
-  const int nch = (v1 - v0 + kSChunkVec - 1) / kSChunkVec;
+  const int nch = (v1 - v0 + kWChunkVec - 1) / kWChunkVec;  // chunks of the span
   volatile int* abort = &sh.abort;
+  volatile float* pub = sh.theta;
 
-  float m_cta = -INFINITY, s_cta = 0.f, t_cta = 0.f;
-  int got = 0;
-  if (warp == kSWarps) {
-    // ------------------------------------------------------------ producer
+  // claim the next chunk of the span and start its copy into ring slot s (lane 0);
+  // returns the chunk, >= nch when none is left
+  auto claim = [&](int s) -> int {
+    int c = nch;
     if (lane == 0) {
-      int c = 0;
-      for (; c < nch; ++c) {
-        const int st = c % kSStages;
-        if (c >= kSStages && !mbar_wait(&sh.empty[st], (c / kSStages - 1) & 1, abort)) {
-          *abort = 1;
-          report(a.dev_status, PRESTO_DEV_TIMEOUT);
-          break;
-        }
-        const int vb = v0 + c * kSChunkVec;
-        const int nv = min(kSChunkVec, v1 - vb);
-        mbar_arrive_expect_tx(&sh.full[st], static_cast<uint32_t>(nv) * 16u);
-        bulk_g2s(ring + st * kSChunkBytes, vecp + vb, static_cast<uint32_t>(nv) * 16u,
-                 &sh.full[st]);
+      c = atomicAdd(&sh.next, 1);
+      if (c < nch) {
+        const int vb = v0 + c * kWChunkVec;
+        const uint32_t bytes = static_cast<uint32_t>(min(kWChunkVec, v1 - vb)) * 16u;
+        mbar_arrive_expect_tx(&sh.full[warp][s], bytes);
+        bulk_g2s(ring + s * kWChunkBytes, vecp + vb, bytes, &sh.full[warp][s]);
       }
-      // no copy may still be landing when the CTA exits (the consumers have waited
-      // for every one already unless they gave up)
-      for (int c2 = c > kSStages ? c - kSStages : 0; c2 < c; ++c2)
-        mbar_wait(&sh.full[c2 % kSStages], (c2 / kSStages) & 1, nullptr);
     }
-  } else {
-    // ------------------------------------------------------------ consumers
-    // extra scalar element: threads 0-6 of part 0 take the head, 8-14 of the last
-    // part the tail (each < 8 elements), with the first chunk
-    int xid = -1;
-    if (part == 0 && tid < head) xid = tid;
-    if (part == a.parts - 1 && tid >= 8 && tid - 8 < V - tail0) xid = tail0 + (tid - 8);
-    const float xval0 = xid >= 0 ? E::load(rowp + xid) : -INFINITY;
-    float mt = -INFINITY, st = 0.f, tt = 0.f;  // running max (plain), Σ 2^u, Σ 2^u u
-    float theta = -INFINITY;                   // candidates: value >= theta ...
-    unsigned long long thr = 1ull;             // ... and key >= thr (every real key is >= 1)
-    int base = 0;                              // candidates kept from earlier chunks
-    const int nloop = nch > 0 ? nch : 1;       // one round for the scalars alone
-    for (int c = 0; c < nloop; ++c) {
-      const int sg = c % kSStages;
-      const int vb = v0 + c * kSChunkVec;
-      const int nv = c < nch ? min(kSChunkVec, v1 - vb) : 0;
-      bool ok = true;
-      if (c < nch && !mbar_wait(&sh.full[sg], (c / kSStages) & 1, abort)) {
-        ok = false;
+    return __shfl_sync(kFull, c, 0);
+  };
+  // the warp's queue: chunks q0, q1, q2 are in flight in slots j, j + 1, j + 2
+  // (mod kWStages), j = chunks taken so far
+  int q0 = claim(0);
+  int q1 = claim(1);
+  int q2 = claim(2);
+  int j = 0;
+
+  float theta = -INFINITY;                   // candidates: value >= theta ...
+  unsigned long long thr = 0ull;             // ... and key > thr, the warp's k-th key
+  unsigned long long lst = 0ull;             // lane j < k: the warp's j-th key
+
+  // one candidate of each lane (key 0: none) at a time through the warp's list
+  auto drain = [&](unsigned& m, auto key_of) {
+    for (unsigned w = __ballot_sync(kFull, m != 0u); w; w = __ballot_sync(kFull, m != 0u)) {
+      const int src = __ffs(w) - 1;
+      const unsigned long long mine = m ? key_of(__ffs(m) - 1) : 0ull;
+      const unsigned long long key = __shfl_sync(kFull, mine, src);
+      if (lane == src) m &= m - 1u;
+      if (key > thr) {
+        thr = warp_insert(lst, key, k, lane);
+        if (thr) {
+          const float tv = key_value(thr);
+          if (tv > theta) {
+            theta = tv;
+            if (lane == 0) pub[warp] = tv;
+          }
+        }
+      }
+    }
+  };
+  // the chunk at the head of the queue (q0 < nch): wait for its copy, take it into
+  // registers and refill its slot with a new claim; false (for the whole warp) when
+  // the wait gave up
+  auto take = [&](uint4 (&d)[kWVec], int& c) -> bool {
+    const int s = j % kWStages;
+    const bool ok = mbar_wait(&sh.full[warp][s], (j / kWStages) & 1, abort);
+    if (!__all_sync(kFull, ok)) {
+      if (lane == 0) {
         *abort = 1;
         report(a.dev_status, PRESTO_DEV_TIMEOUT);
       }
-      uint4 d[kSVec];
-      const uint32_t ni = E::kNegInfWord;
-      auto load_chunk = [&]() {
-#pragma unroll
-        for (int i = 0; i < kSVec; ++i) {
-          const int vi = i * kSCons + tid;
-          d[i] = (ok && vi < nv)
-                     ? *reinterpret_cast<const uint4*>(ring + sg * kSChunkBytes + vi * 16)
-                     : make_uint4(ni, ni, ni, ni);
-        }
-      };
-      load_chunk();  // the slot is released once the chunk's candidates are taken
-      const float xval = c == 0 ? xval0 : -INFINITY;
-      const bool xin = c == 0 && xid >= 0;
-
-      // ---- the chunk's maximum and the online (max, Σ 2^u) pair, log2 domain
-      float cm = xval;
-#pragma unroll
-      for (int i = 0; i < kSVec; ++i) cm = fmaxf(cm, E::vmax(d[i]));
-      if (cm > mt) {
-        if (mt != -INFINITY) {
-          const float dl = mt * kLog2e - cm * kLog2e;  // the old reference minus the new
-          const float f = ex2(dl);
-          if constexpr (ENT) tt = f * fmaf(dl, st, tt);
-          st *= f;
-        }
-        mt = cm;
-      }
-      if (mt != -INFINITY) {
-        const float m2 = mt * kLog2e;
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
-        if constexpr (!ENT) {
-#pragma unroll
-          for (int i = 0; i < kSVec; ++i)
-#pragma unroll
-            for (int e = 0; e < n; ++e) acc[e & 3] += ex2(fmaf(E::value(d[i], e), kLog2e, -m2));
-          if (xin) acc[0] += ex2(fmaf(xval, kLog2e, -m2));
-        } else {
-          // u clamped at -256: 2^u flushes to 0 there, so -inf adds 0 to both sums
-          float tac[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-          for (int i = 0; i < kSVec; ++i)
-#pragma unroll
-            for (int e = 0; e < n; ++e) {
-              const float u = fmaxf(fmaf(E::value(d[i], e), kLog2e, -m2), -256.f);
-              const float p = ex2(u);
-              acc[e & 3] += p;
-              tac[e & 3] = fmaf(p, u, tac[e & 3]);
-            }
-          if (xin) {
-            const float u = fmaxf(fmaf(xval, kLog2e, -m2), -256.f);
-            const float p = ex2(u);
-            acc[0] += p;
-            tac[0] = fmaf(p, u, tac[0]);
-          }
-          tt += (tac[0] + tac[1]) + (tac[2] + tac[3]);
-        }
-        st += (acc[0] + acc[1]) + (acc[2] + acc[3]);
-      }
-
-      // ---- first chunk: theta = the k-th largest half-warp maximum (CTA-wide, once)
-      if (c == 0) {
-        float hm = cm;
-#pragma unroll
-        for (int off = 8; off > 0; off >>= 1) hm = fmaxf(hm, __shfl_xor_sync(kFull, hm, off));
-        if ((lane & 15) == 0) sh.gmax[warp * 2 + (lane >> 4)] = hm;
-        consumers_sync();
-        if (warp == 0 && lane < 2 * kSWarps) {
-          const float x = sh.gmax[lane];
-          int r = 0;
-#pragma unroll
-          for (int u = 0; u < 2 * kSWarps; ++u) {
-            const float y = sh.gmax[u];
-            r += y > x || (y == x && u < lane);
-          }
-          if (r == k - 1) sh.theta = x;
-        }
-        consumers_sync();
-        theta = sh.theta;
-      } else {
-        // later chunks: every warp publishes its half-warps' running maxima (real
-        // elements, so the k-th largest of the 16 published values still has k
-        // elements at or above it) and raises its own threshold to that k-th largest,
-        // with no barrier: a value another warp has not yet raised is only a looser
-        // bound
-        volatile float* gm = sh.gmax;
-        float hm = mt;
-#pragma unroll
-        for (int off = 8; off > 0; off >>= 1) hm = fmaxf(hm, __shfl_xor_sync(kFull, hm, off));
-        if ((lane & 15) == 0) gm[warp * 2 + (lane >> 4)] = hm;
-        __syncwarp();
-        const float x = lane < 2 * kSWarps ? gm[lane] : -INFINITY;
-        int r = 0;
-#pragma unroll
-        for (int u = 0; u < 2 * kSWarps; ++u) {
-          const float y = __shfl_sync(kFull, x, u);
-          r += y > x || (y == x && u < lane);
-        }
-        const unsigned who = __ballot_sync(kFull, lane < 2 * kSWarps && r == k - 1);
-        theta = fmaxf(theta, __shfl_sync(kFull, x, __ffs(who) - 1));
-      }
-
-      // ---- candidates of the chunk (value >= theta, key >= thr), appended one by one
-      // (they are rare) at base + a per-chunk counter.  The counter of chunk c + 2
-      // is cleared right after chunk c's barrier: every thread read it (as chunk
-      // c - 1's) before that barrier, and appends to it only after the next one.
-      auto emit_chunk = [&](unsigned long long thr_k, int* ctr, int at) {
-#pragma unroll
-        for (int i = 0; i < kSVec; ++i) {
-          const int vi = i * kSCons + tid;
-          if (vi < nv && E::vmax(d[i]) >= theta) {
-            const int id0 = head + (vb + vi) * n;
-#pragma unroll
-            for (int e = 0; e < n; ++e) {
-              const float x = E::value(d[i], e);
-              const unsigned long long key = elem_key(x, id0 + e);
-              if (x >= theta && key >= thr_k) {
-                const int j = at + atomicAdd(ctr, 1);
-                if (j < kSCap) sh.cand2[j] = key;
-              }
-            }
-          }
-        }
-        if (xin && xval >= theta) {
-          const unsigned long long key = elem_key(xval, xid);
-          if (key >= thr_k) {
-            const int j = at + atomicAdd(ctr, 1);
-            if (j < kSCap) sh.cand2[j] = key;
-          }
-        }
-      };
-      const int cs = c % 3;
-      emit_chunk(thr, &sh.cnt[cs], base);
-      if (tid == 0) sh.stop[c & 1] = *abort;  // one reading for all consumers
-      consumers_sync();
-      int M = base + sh.cnt[cs];
-      const int stop = sh.stop[c & 1];
-      if (tid == 0) sh.cnt[(c + 2) % 3] = 0;
-      while (M > kSCap) {
-        // overflow: the k-th largest of the buffer's keys bounds the span's top-k
-        // from below; keep the earlier chunks' keys above it and re-scan this one
-        rank_keys<kSCons>(sh.cand2, kSCap, k, sh.list, tid);
-        consumers_sync();
-        thr = sh.list[k - 1];
-        unsigned long long keep[kSCompact / kSCons];
-#pragma unroll
-        for (int j = 0; j < kSCompact / kSCons; ++j) {
-          const int e = j * kSCons + tid;
-          keep[j] = (e < base && sh.cand2[e] >= thr) ? sh.cand2[e] : 0ull;
-        }
-        if (tid == 0) sh.fcnt = 0;
-        consumers_sync();
-#pragma unroll
-        for (int j = 0; j < kSCompact / kSCons; ++j)
-          if (keep[j]) sh.cand2[atomicAdd(&sh.fcnt, 1)] = keep[j];
-        consumers_sync();
-        base = sh.fcnt;
-        consumers_sync();
-        if (tid == 0) sh.fcnt = 0;
-        consumers_sync();
-        load_chunk();  // the chunk again, from its ring slot
-        emit_chunk(thr, &sh.fcnt, base);
-        consumers_sync();
-        M = base + sh.fcnt;
-        consumers_sync();  // every thread has read the counter
-      }
-      __syncwarp();
-      if (c < nch && lane == 0) mbar_arrive(&sh.empty[sg]);  // the slot may be refilled
-      if (M > kSCompact) {
-        // cut back to the running top-k and raise the thresholds to its k-th key
-        rank_keys<kSCons>(sh.cand2, M, k, sh.list, tid);
-        consumers_sync();
-        thr = sh.list[k - 1];
-        if (tid < k) sh.cand2[tid] = sh.list[tid];
-        M = k;
-        consumers_sync();
-      }
-      if (thr > 1ull) theta = fmaxf(theta, key_value(thr));
-      base = M;
-      if (stop) break;
+      return false;
     }
-    // ---- the span's top-k and its (max, sum) pair
-    rank_keys<kSCons>(sh.cand2, base, k, sh.list, tid);
-    got = base < k ? base : k;
-    const uint32_t wm_o = __reduce_max_sync(kFull, ordered(mt));
-    const float wm = unordered(wm_o);
-    const float wm2 = wm * kLog2e;
-    const float m2 = mt * kLog2e;
-    const float fw = (mt == -INFINITY) ? 0.f : ex2(m2 - wm2);
-    float ws = st * fw;
+    c = q0;
+    const int nv = min(kWChunkVec, v1 - (v0 + c * kWChunkVec));
+    const uint32_t ni = E::kNegInfWord;
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) ws += __shfl_xor_sync(kFull, ws, off);
-    float wt = 0.f;
-    if constexpr (ENT) {
-      wt = (mt == -INFINITY) ? 0.f : fw * fmaf(m2 - wm2, st, tt);
+    for (int i = 0; i < kWVec; ++i) {
+      const int vi = i * 32 + lane;
+      d[i] = vi < nv ? *reinterpret_cast<const uint4*>(ring + s * kWChunkBytes + vi * 16)
+                     : make_uint4(ni, ni, ni, ni);
+    }
+    __syncwarp();
+    if (lane == 0) fence_proxy_async();  // the slot's reads come before its refill
+    const int qn = claim(s);
+    q0 = q1;
+    q1 = q2;
+    q2 = qn;
+    ++j;
+    return true;
+  };
+  // chunk c: the lane's maximum (returned), and the chunk's (max log2, Σ 2^u[, Σ 2^u u])
+  // summed over the warp in a fixed order into slot c; eight accumulators a lane
+  auto reduce = [&](const uint4 (&d)[kWVec], int c) -> float {
+    const float cm = E::template max_of<kWVec>(d);
+    const float mw = unordered(__reduce_max_sync(kFull, ordered(cm)));
+    float sc = 0.f, tc = 0.f;
+    if (mw != -INFINITY) {
+      const float m2 = mw * kLog2e;
+      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      if constexpr (!ENT) {
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) wt += __shfl_xor_sync(kFull, wt, off);
+        for (int i = 0; i < kWVec; ++i)
+#pragma unroll
+          for (int e = 0; e < n; ++e)
+            acc[(i * n + e) & 7] += ex2(fmaf(E::value(d[i], e), kLog2e, -m2));
+      } else {
+        // u clamped at -256: 2^u flushes to 0 there, so -inf adds 0 to both sums
+        float tac[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < kWVec; ++i)
+#pragma unroll
+          for (int e = 0; e < n; ++e) {
+            const float u = fmaxf(fmaf(E::value(d[i], e), kLog2e, -m2), -256.f);
+            const float p = ex2(u);
+            acc[(i * n + e) & 7] += p;
+            tac[(i * n + e) & 7] = fmaf(p, u, tac[(i * n + e) & 7]);
+          }
+        tc = ((tac[0] + tac[1]) + (tac[2] + tac[3])) + ((tac[4] + tac[5]) + (tac[6] + tac[7]));
+      }
+      sc = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      sc += __shfl_xor_sync(kFull, sc, off);
+      if constexpr (ENT) tc += __shfl_xor_sync(kFull, tc, off);
     }
     if (lane == 0) {
-      sh.warp_ms[warp] = make_float2(wm == -INFINITY ? -INFINITY : wm2, ws);
-      if constexpr (ENT) sh.warp_t[warp] = wt;
+      sh.cms[c] = make_float2(mw == -INFINITY ? -INFINITY : mw * kLog2e, sc);
+      if constexpr (ENT) sh.cts[c] = tc;
     }
-    consumers_sync();
-    if (warp == 0) {
-      float mw = lane < kSWarps ? sh.warp_ms[lane].x : -INFINITY;
-      float sw = lane < kSWarps ? sh.warp_ms[lane].y : 0.f;
-      float tw = 0.f;
-      if constexpr (ENT) tw = lane < kSWarps ? sh.warp_t[lane] : 0.f;
+    return cm;
+  };
+  // theta = the best k-th value any warp of the CTA has published so far
+  auto refresh = [&]() {
+    float tp = lane < kWWarps ? pub[lane] : -INFINITY;
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const float m_o = __shfl_xor_sync(kFull, mw, off);
-        const float s_o = __shfl_xor_sync(kFull, sw, off);
-        if constexpr (ENT) {
-          const float t_o = __shfl_xor_sync(kFull, tw, off);
-          merge_mst(mw, sw, tw, m_o, s_o, t_o);
-        } else {
-          merge_ms(mw, sw, m_o, s_o);
-        }
+    for (int off = 4; off > 0; off >>= 1) tp = fmaxf(tp, __shfl_xor_sync(kFull, tp, off));
+    theta = fmaxf(theta, __shfl_sync(kFull, tp, 0));
+  };
+  // candidates of chunk c (cm: the lane's chunk maximum; padding vectors hold -inf
+  // and are never taken)
+  auto collect = [&](const uint4 (&d)[kWVec], float cm, int c) {
+    const bool lane_hit = cm >= theta;
+    if (!__any_sync(kFull, lane_hit)) return;
+    const int vb = v0 + c * kWChunkVec;
+    const int nv = min(kWChunkVec, v1 - vb);
+    unsigned hits = 0u;
+    if (lane_hit) {
+#pragma unroll
+      for (int i = 0; i < kWVec; ++i)
+        if (i * 32 + lane < nv && E::vmax(d[i]) >= theta) hits |= 1u << i;
+    }
+    if (!__any_sync(kFull, hits != 0u)) return;
+#pragma unroll
+    for (int i = 0; i < kWVec; ++i) {
+      if (!__any_sync(kFull, (hits >> i) & 1u)) continue;
+      unsigned m = 0u;
+      if ((hits >> i) & 1u) {
+#pragma unroll
+        for (int e = 0; e < n; ++e)
+          if (E::value(d[i], e) >= theta) m |= 1u << e;
       }
-      m_cta = mw;
-      s_cta = sw;
-      t_cta = tw;
+      const int id0 = head + (vb + i * 32 + lane) * n;
+      const uint4 di = d[i];
+      drain(m, [&](int e) { return elem_key(E::value(di, e), id0 + e); });
+    }
+  };
+
+  // ---- every warp's first chunk, then the CTA's first threshold: the k-th largest
+  // of all lanes' first-chunk maxima (as ordered integers; -inf where a lane had no
+  // data).  Each warp's k largest come from k warp-wide maximum reductions; then a
+  // thread per value counts the larger ones.
+  uint4 d[kWVec];
+  bool alive = true;
+  float cm0 = -INFINITY;
+  int c0 = -1;
+  if (q0 < nch) {
+    alive = take(d, c0);
+    if (alive) cm0 = reduce(d, c0);
+  }
+  {
+    uint32_t o = ordered(cm0);  // >= ordered(-inf) > 0: a taken lane's 0 never wins
+    for (int s2 = 0; s2 < k; ++s2) {
+      const uint32_t mx = __reduce_max_sync(kFull, o);
+      if (lane == 0) sh.first[warp * k + s2] = mx;
+      const unsigned win = __ballot_sync(kFull, o == mx);
+      if (lane == __ffs(win) - 1) o = 0u;
     }
   }
-  __syncthreads();  // producer and consumers
-  finish_row<ENT, kSCons>(a, sh, row, part, m_cta, s_cta, t_cta, got);
+  __syncthreads();
+  if (tid < kWWarps * k) {
+    const uint32_t v = sh.first[tid];
+    const int nf = kWWarps * k;
+    int r = 0;
+    int u = 0;
+    for (; u + 8 <= nf; u += 8) {
+#pragma unroll
+      for (int z = 0; z < 8; ++z) {
+        const uint32_t y = sh.first[u + z];
+        r += y > v || (y == v && u + z < tid);
+      }
+    }
+    for (; u < nf; ++u) {
+      const uint32_t y = sh.first[u];
+      r += y > v || (y == v && u < tid);
+    }
+    if (r == k - 1) sh.theta0 = unordered(v);
+  }
+  __syncthreads();
+  theta = sh.theta0;
+  if (lane == 0 && theta > pub[warp]) pub[warp] = theta;
+
+  // ---- the chunks
+  if (alive && c0 >= 0) collect(d, cm0, c0);
+  while (alive && q0 < nch) {
+    int c;
+    if (!take(d, c)) {
+      alive = false;
+      break;
+    }
+    const float cm = reduce(d, c);
+    refresh();
+    collect(d, cm, c);
+  }
+  if (!alive && lane == 0) {
+    // gave up: no copy of this warp may still be landing when the CTA exits
+    const int q[kWStages] = {q0, q1, q2};
+    for (int u = 0; u < kWStages; ++u)
+      if (q[u] < nch)
+        mbar_wait(&sh.full[warp][(j + u) % kWStages], ((j + u) / kWStages) & 1, nullptr);
+  }
+
+  // ---- scalar elements (warp 0): the head of part 0 (lanes 0-6) and the tail of
+  // the last part (lanes 8-14), each < 8 elements; their pair goes to slot nch
+  if (warp == 0) {
+    int xid = -1;
+    if (part == 0 && lane < head) xid = lane;
+    if (part == a.parts - 1 && lane >= 8 && lane - 8 < V - tail0) xid = tail0 + (lane - 8);
+    const float x = xid >= 0 ? E::load(rowp + xid) : -INFINITY;
+    float m2 = x * kLog2e, sx = 0.f, tx = 0.f;
+    if (xid >= 0 && x != -INFINITY) sx = 1.f;  // 2^(x log2e - m2) = 1, u = 0
+    else m2 = -INFINITY;
+    warp_merge_pairs<ENT>(m2, sx, tx);
+    if (lane == 0) {
+      sh.cms[nch] = make_float2(m2, sx);
+      if constexpr (ENT) sh.cts[nch] = tx;
+    }
+    refresh();
+    unsigned m = (xid >= 0 && x >= theta) ? 1u : 0u;
+    drain(m, [&](int) { return elem_key(x, xid); });
+  }
+
+  // ---- every warp's keys at or above theta, and the CTA's (max, Σ) pair from its
+  // chunks' pairs in chunk order, into the leader
+  refresh();
+  WSmem* ld = &sh;
+  if (a.parts > 1) ld = cg::this_cluster().map_shared_rank(&sh, 0);
+  if (lane < k)
+    ld->keys[(part * kWWarps + warp) * k + lane] =
+        (lst != 0ull && key_value(lst) >= theta) ? lst : 0ull;
+  __syncthreads();  // every chunk's pair is in place
+  if (warp == 0) {
+    // lane l folds pairs l, l + 32, ... in order; then the warp merges the lanes
+    float M = -INFINITY;
+    for (int c = lane; c <= nch; c += 32) M = fmaxf(M, sh.cms[c].x);
+    M = unordered(__reduce_max_sync(kFull, ordered(M)));
+    float sp = 0.f, tp = 0.f;
+    if (M != -INFINITY) {
+      for (int c = lane; c <= nch; c += 32) {
+        const float2 p = sh.cms[c];
+        if (p.x == -INFINITY) continue;
+        const float f = ex2(p.x - M);
+        sp = fmaf(p.y, f, sp);
+        if constexpr (ENT) tp = fmaf(f, fmaf(p.x - M, p.y, sh.cts[c]), tp);
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      sp += __shfl_xor_sync(kFull, sp, off);
+      if constexpr (ENT) tp += __shfl_xor_sync(kFull, tp, off);
+    }
+    if (lane == 0) {
+      ld->ms[part] = make_float2(M, sp);
+      if constexpr (ENT) ld->ts[part] = tp;
+    }
+  }
+  if (a.parts > 1)
+    cg::this_cluster().sync();
+  else
+    __syncthreads();
+  if (part != 0) return;
+
+  // ---- leader: the row's top-k among the kept keys (every one of the row's top-k is
+  // kept, so at least k are real), and its (max, Σ) from the warps' pairs
+  const int M = a.parts * kWWarps * k;
+  for (int i = tid; i < M; i += kWThreads) {
+    const unsigned long long ki = sh.keys[i];
+    if (ki == 0ull) continue;
+    int r = 0;
+    int u = 0;
+    for (; u + 8 <= M; u += 8) {
+#pragma unroll
+      for (int z = 0; z < 8; ++z) r += sh.keys[u + z] > ki;
+    }
+    for (; u < M; ++u) r += sh.keys[u] > ki;
+    if (r < k) sh.list[r] = ki;
+  }
+  float m_row = -INFINITY, s_row = 0.f, t_row = 0.f;
+  if (warp == 0) {
+    m_row = lane < a.parts ? sh.ms[lane].x : -INFINITY;
+    s_row = lane < a.parts ? sh.ms[lane].y : 0.f;
+    if constexpr (ENT) t_row = lane < a.parts ? sh.ts[lane] : 0.f;
+    warp_merge_pairs<ENT>(m_row, s_row, t_row);
+  }
+  __syncthreads();  // the row's list is complete
+  if (warp == 0) write_row<ENT>(a, sh.list, row, m_row, s_row, t_row);
 }
 
 template <typename T, int VMAX, bool ENT>
@@ -958,11 +1063,11 @@ Plan make_plan(int B, int L, int V, int elem_bytes, bool ent) {
   // per SM or more (a row's spans still form one cluster of <= 8 CTAs)
   const int act = active_clusters(elem_bytes, p.vmax, p.parts, ent);
   if (act >= 1 && p.rows > act) {
-    const int sms = sm_count();
-    int parts = (sms + p.rows - 1) / p.rows;
+    const int slots = kWCtasPerSm * sm_count();  // resident CTAs of the streaming kernel
+    int parts = slots / p.rows;
     parts = parts < 1 ? 1 : (parts > kMaxParts ? kMaxParts : parts);
     const int nv = V / p.epv;  // a row's aligned vectors, up to one
-    while (parts > 1 && (nv + parts - 1) / parts < kSChunkVec / 2) --parts;  // no tiny spans
+    while (parts > 1 && (nv + parts - 1) / parts < kWWarps * kWChunkVec / 2) --parts;  // no tiny spans
     p.stream = true;
     p.parts = parts;
     p.vpt = (nv + 1 + parts - 1) / parts;
@@ -991,12 +1096,12 @@ template <typename T, bool ENT>
 cudaError_t launch_stream(const Plan& p, const Args& a, cudaStream_t stream) {
   static const cudaError_t attr = cudaFuncSetAttribute(
       topk_stream_kernel<T, ENT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-      static_cast<int>(kSDynBytes));
+      static_cast<int>(kWDynBytes));
   if (attr != cudaSuccess) return attr;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(p.rows) * p.parts);
-  cfg.blockDim = dim3(kSThreads);
-  cfg.dynamicSmemBytes = kSDynBytes;
+  cfg.blockDim = dim3(kWThreads);
+  cfg.dynamicSmemBytes = kWDynBytes;
   cfg.stream = stream;
   cudaLaunchAttribute at[2];
   at[0].id = cudaLaunchAttributeClusterDimension;

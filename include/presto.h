@@ -108,28 +108,6 @@ int presto_topk(const void* logits, int dtype, int B, int L, int V, long long ro
                 size_t ws_bytes, int32_t* dev_status, presto_stream_t stream);
 
 /*
- * presto_topk_noalloc - presto_topk for callers that cannot allocate device memory.
- * The paper has no counterpart; this is a deployment variant of presto_topk.
- *
- * Same arguments and results as presto_topk, without the workspace: whatever
- * scratch the plan needs lives in a file-scope device array of
- * PRESTO_TOPK_STATIC_SCRATCH_BYTES (16 KiB) that every GPU loading this library
- * keeps for the life of the process.  Returns PRESTO_ERR_UNSUPPORTED, enqueueing
- * nothing, when presto_topk_workspace(B, L, V, k) exceeds that size (no shape does
- * with the current plan).  Calls no cudaMalloc or
- * cudaFree.  The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress, with that device current) and caches it; make that
- * first call before any stream capture.  All calls on a device share the one
- * array, so calls whose kernels may overlap on the GPU race; order them on one
- * stream.  The array keeps the last call's contents; the call clears what must
- * start at zero on `stream` itself.
- */
-#define PRESTO_TOPK_STATIC_SCRATCH_BYTES (1u << 14)
-int presto_topk_noalloc(const void* logits, int dtype, int B, int L, int V,
-                        long long row_stride, int k, int32_t* topk_ids, float* topk_logq,
-                        float* lse, int32_t* dev_status, presto_stream_t stream);
-
-/*
  * presto_topk_entropy - presto_topk that also yields each row's entropy and the
  * entropy-adaptive lambda_d of App. F, in the same single pass over the logits.
  *
@@ -312,6 +290,44 @@ int presto_score_build_tree_mask(const int32_t* topk_ids, const float* topk_logq
                                  const int32_t* kv_len, uint32_t* mask, int32_t* pos_ids,
                                  void* ws, size_t ws_bytes, int32_t* dev_status,
                                  presto_stream_t stream);
+
+/*
+ * presto_score_build_tree_noalloc - presto_score_build_tree_mask for callers that
+ * cannot allocate device memory.  The paper has no counterpart: this is a
+ * deployment variant of the same kernel.
+ *
+ * Some callers have no way to hand this library a workspace: a plugin inside a
+ * serving framework whose allocator owns all of the GPU's memory, a C program with
+ * no allocator at all, or a latency-critical loop that must never block in
+ * cudaMalloc (which can synchronise the device and can fail once memory is
+ * fragmented).  Large node budgets (N = 512, 1024) make the tree build keep its
+ * level-selection scratch and child tables in global memory; this entry point keeps
+ * them in a fixed device array inside the library instead, of
+ * PRESTO_BUILD_STATIC_SCRATCH_BYTES (1 MiB).  Every GPU that loads the library
+ * holds that array until the process exits.  It fits, for example, two sequences at
+ * N = 1024 (k = b = 8, with a trigram table) or sixteen at N = 512.
+ *
+ * Arguments and results are those of presto_score_build_tree_mask without ws and
+ * ws_bytes.  Returns PRESTO_ERR_UNSUPPORTED, enqueueing nothing, when the call
+ * needs more scratch than the array holds (B times the per-sequence need of the
+ * shape; see presto_build_workspace_ex).  Calls no cudaMalloc, cudaFree or other
+ * allocating routine.  The first call on a device looks up the array's device
+ * address (cudaGetSymbolAddress, with that device current) and caches it; make that
+ * first call before any stream capture.  All calls on a device share the one array
+ * and it keeps the last call's contents; nothing in it has to start at zero (every
+ * call writes each scratch entry before reading it).  Calls whose kernels may
+ * overlap on the GPU (different streams with no ordering between them) race on the
+ * array: order them on one stream.
+ */
+#define PRESTO_BUILD_STATIC_SCRATCH_BYTES (1u << 20)
+int presto_score_build_tree_noalloc(const int32_t* topk_ids, const float* topk_logq, int B,
+                                    int L, int k, int b, const int32_t* ctx2,
+                                    const presto_ngram3* ngram, float lambda,
+                                    const float* lambda_d, int policy, int beam_width, int N,
+                                    int32_t* node_token, int32_t* node_parent,
+                                    int32_t* node_depth, float* node_score, int32_t* n_nodes,
+                                    const int32_t* kv_len, uint32_t* mask, int32_t* pos_ids,
+                                    int32_t* dev_status, presto_stream_t stream);
 
 /*
  * presto_tree_mask - tree attention mask and position ids (§4.3 and App. C (I),

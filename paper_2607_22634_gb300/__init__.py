@@ -21,9 +21,9 @@ from ._lib import (  # noqa: F401
     presto_attn_workspace,
     presto_build_workspace,
     presto_score_build_tree,
+    presto_score_build_tree_noalloc,
     presto_topk,
     presto_topk_entropy,
-    presto_topk_noalloc,
     presto_topk_slots,
     presto_topk_workspace,
     presto_tree_attention,

@@ -47,7 +47,6 @@ _SIGS = {
     "presto_topk_workspace": (ctypes.c_size_t, [_I, _I, _I, _I]),
     "presto_topk": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, _P, _P, _P, _P,
                          ctypes.c_size_t, _P, _P]),
-    "presto_topk_noalloc": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, _P, _P, _P, _P, _P]),
     "presto_topk_slots": (_I, [_P, _I, _I, _I, _I, _I, ctypes.c_longlong, _P, _P, _I, _I, _I, _I,
                                _P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "presto_topk_entropy": (_I, [_P, _I, _I, _I, _I, ctypes.c_longlong, _I, ctypes.c_float,
@@ -62,6 +61,9 @@ _SIGS = {
     "presto_score_build_tree_mask": (_I, [_P, _P, _I, _I, _I, _I, _P, ctypes.POINTER(Ngram3),
                                           ctypes.c_float, _P, _I, _I, _I, _P, _P, _P, _P, _P,
                                           _P, _P, _P, _P, ctypes.c_size_t, _P, _P]),
+    "presto_score_build_tree_noalloc": (_I, [_P, _P, _I, _I, _I, _I, _P,
+                                             ctypes.POINTER(Ngram3), ctypes.c_float, _P, _I, _I,
+                                             _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P]),
     "presto_score_build_tree": (_I, [_P, _P, _I, _I, _I, _I, _P, ctypes.POINTER(Ngram3),
                                      ctypes.c_float, _I, _P, _P, _P, _P, _P, _P,
                                      ctypes.c_size_t, _P, _P]),
@@ -160,24 +162,6 @@ def presto_topk(logits, k, topk_ids=None, topk_logq=None, lse=None, ws=None, dev
                             _ptr(topk_logq), _ptr(lse), _ptr(ws), nws, _ptr(dev_status),
                             _stream(stream))
     _check(st, "presto_topk")
-    return topk_ids, topk_logq, lse
-
-
-def presto_topk_noalloc(logits, k, topk_ids, topk_logq, lse=None, dev_status=None, stream=None):
-    """presto_topk without a workspace: for callers that must not allocate device
-    memory.  The library keeps the scratch in a fixed 16 KiB device array shared
-    by every call on the device, so calls that may overlap on the GPU race.
-    Outputs must be passed in (nothing is allocated here either)."""
-    B, L, V = logits.shape
-    dtype = {torch.float32: PRESTO_F32, torch.bfloat16: PRESTO_BF16}.get(logits.dtype)
-    if dtype is None or logits.stride(2) != 1:
-        raise ValueError("logits must be float32 or bfloat16 with unit last stride")
-    _need(topk_ids, torch.int32, (B, L, k), "topk_ids")
-    _need(topk_logq, torch.float32, (B, L, k), "topk_logq")
-    st = load().presto_topk_noalloc(_ptr(logits), dtype, B, L, V, logits.stride(1), k,
-                                    _ptr(topk_ids), _ptr(topk_logq), _ptr(lse), _ptr(dev_status),
-                                    _stream(stream))
-    _check(st, "presto_topk_noalloc")
     return topk_ids, topk_logq, lse
 
 
@@ -360,6 +344,40 @@ def presto_score_build_tree(topk_ids, topk_logq, ctx2, ngram, lam, N, b=None, ou
         _ptr(pos_ids) if kv_len is not None else None, _ptr(ws), nws, _ptr(dev_status),
         _stream(stream))
     _check(st, "presto_score_build_tree_mask")
+    return out
+
+
+def presto_score_build_tree_noalloc(topk_ids, topk_logq, ctx2, ngram, lam, N, out, b=None,
+                                    dev_status=None, stream=None, lambda_d=None,
+                                    policy=SEARCH_BEST_FIRST, beam_width=1, kv_len=None,
+                                    mask=None, pos_ids=None):
+    """presto_score_build_tree without a workspace, for callers that cannot allocate
+    device memory: the library keeps the build's scratch in a fixed 1 MiB device
+    array shared by every call on the device (calls that may overlap on the GPU
+    race).  Outputs are passed in (``out`` as presto_score_build_tree returns it,
+    plus mask and pos_ids with kv_len): nothing is allocated here either."""
+    B, L, k = topk_ids.shape
+    b = k if b is None else b
+    _need(topk_ids, torch.int32, (B, L, k), "topk_ids")
+    _need(topk_logq, torch.float32, (B, L, k), "topk_logq")
+    _need(ctx2, torch.int32, (B, 2), "ctx2")
+    for key, dt, shape in (("token", torch.int32, (B, N)), ("parent", torch.int32, (B, N)),
+                           ("depth", torch.int32, (B, N)), ("score", torch.float32, (B, N)),
+                           ("n_nodes", torch.int32, (B,))):
+        _need(out[key], dt, shape, key)
+    if kv_len is not None:
+        W = (N + 31) // 32
+        _need(kv_len, torch.int32, (B,), "kv_len")
+        _need(mask, torch.int32, (B, N, W), "mask")
+        _need(pos_ids, torch.int32, (B, N), "pos_ids")
+    desc = None if ngram is None else ctypes.byref(ngram.desc)
+    st = load().presto_score_build_tree_noalloc(
+        _ptr(topk_ids), _ptr(topk_logq), B, L, k, b, _ptr(ctx2), desc, float(lam),
+        _ptr(lambda_d), int(policy), int(beam_width), N,
+        _ptr(out["token"]), _ptr(out["parent"]), _ptr(out["depth"]), _ptr(out["score"]),
+        _ptr(out["n_nodes"]), _ptr(kv_len), _ptr(mask), _ptr(pos_ids), _ptr(dev_status),
+        _stream(stream))
+    _check(st, "presto_score_build_tree_noalloc")
     return out
 
 

@@ -1239,64 +1239,3 @@ extern "C" int presto_topk_slots(const void* slot_logits, int dtype, int B, int 
   return topk_common(slot_logits, dtype, B, L, V, row_stride, k, topk_ids, topk_logq, lse,
                      nullptr, nullptr, 0.f, 0.f, &sr, dev_status, stream);
 }
-
-// ---------------------------------------------------------------------------
-// Allocation-free top-k.
-//
-// Some callers cannot hand this library a workspace: a plugin running inside an
-// inference server whose device memory all belongs to the host framework's
-// allocator, a C caller with no allocator handle at all, or a latency-critical
-// loop that must not call cudaMalloc (which can block on device-wide
-// synchronisation and fail under fragmentation).  For them this entry point
-// hands presto_topk a fixed file-scope device array as its workspace, and
-// otherwise runs the same code.  (The current plan merges a row's spans inside a
-// thread-block cluster and uses no workspace, so the array is reserved rather
-// than used.)
-//
-// The array costs kStaticScratchBytes on every GPU that loads this library, for
-// the life of the process.  All calls on one device share it: should a plan use
-// it, two calls whose kernels overlap on the GPU (different streams, no ordering
-// between them) would race on it.
-// ---------------------------------------------------------------------------
-namespace presto {
-namespace {
-
-constexpr size_t kStaticScratchBytes = PRESTO_TOPK_STATIC_SCRATCH_BYTES;
-__device__ __align__(256) unsigned char g_topk_scratch[kStaticScratchBytes];
-
-std::mutex g_scratch_mutex;
-void* g_scratch_addr[64] = {};
-
-// Device address of g_topk_scratch for the current device.  Host code cannot use
-// the symbol itself (its host-side name is only a stand-in), so the address is
-// looked up once per device, with that device current, and cached.
-void* static_scratch() {
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  std::lock_guard<std::mutex> lock(g_scratch_mutex);
-  if (!g_scratch_addr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_topk_scratch) != cudaSuccess || !p) return nullptr;
-    g_scratch_addr[dev] = p;
-  }
-  return g_scratch_addr[dev];
-}
-
-}  // namespace
-}  // namespace presto
-
-extern "C" int presto_topk_noalloc(const void* logits, int dtype, int B, int L, int V,
-                                   long long row_stride, int k, int32_t* topk_ids,
-                                   float* topk_logq, float* lse, int32_t* dev_status,
-                                   presto_stream_t stream) {
-  PRESTO_CHECK_ARG(logits && topk_ids && topk_logq);
-  PRESTO_CHECK_ARG(dtype == PRESTO_F32 || dtype == PRESTO_BF16);
-  PRESTO_CHECK_ARG(B >= 1 && L >= 1 && V >= 1 && k >= 1 && k <= V && row_stride >= V);
-  PRESTO_CHECK_LIMIT(k <= kMaxK && V < kMaxV && L <= kMaxL);
-  const size_t need = presto_topk_workspace(B, L, V, k);
-  if (need > kStaticScratchBytes) return PRESTO_ERR_UNSUPPORTED;
-  void* ws = static_scratch();
-  if (!ws) return PRESTO_ERR_CUDA;
-  return presto_topk(logits, dtype, B, L, V, row_stride, k, topk_ids, topk_logq, lse, ws,
-                     kStaticScratchBytes, dev_status, stream);
-}

@@ -20,6 +20,7 @@
 #include <cooperative_groups.h>
 
 #include <initializer_list>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -983,4 +984,69 @@ extern "C" int presto_score_build_tree_mask(
   cfg.numAttrs = 2;
   if (cudaLaunchKernelEx(&cfg, build_kernel, a) != cudaSuccess) return PRESTO_ERR_CUDA;
   return launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free tree build.
+//
+// For callers that cannot hand the library a workspace: a plugin inside a serving
+// framework whose allocator owns all of the GPU's memory, a C program with no
+// allocator, or a latency-critical loop that must never block in cudaMalloc.  Large
+// node budgets keep the selection scratch and child tables in global memory; here
+// they live in a fixed file-scope device array instead, and the build otherwise runs
+// exactly as presto_score_build_tree_mask.  The array costs
+// PRESTO_BUILD_STATIC_SCRATCH_BYTES on every GPU that loads the library, for the
+// life of the process.  All calls on a device share it and it keeps the last call's
+// contents: the kernel writes every scratch entry it reads before reading it, so
+// nothing has to be cleared, and two calls whose kernels overlap on the GPU (no
+// ordering between their streams) race on it.
+// ---------------------------------------------------------------------------
+namespace presto {
+namespace {
+
+constexpr size_t kBuildStaticScratch = PRESTO_BUILD_STATIC_SCRATCH_BYTES;
+__device__ __align__(256) unsigned char g_build_scratch[kBuildStaticScratch];
+
+std::mutex g_build_scratch_mutex;
+void* g_build_scratch_addr[64] = {};
+
+// Device address of g_build_scratch on the current device.  In host code the
+// symbol's name is only a host-side stand-in, so the address is looked up once per
+// device, with that device current, and cached; nullptr when the lookup fails.
+void* build_static_scratch() {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(g_build_scratch_mutex);
+  if (!g_build_scratch_addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_build_scratch) != cudaSuccess || !p) {
+      cudaGetLastError();
+      return nullptr;
+    }
+    g_build_scratch_addr[dev] = p;
+  }
+  return g_build_scratch_addr[dev];
+}
+
+}  // namespace
+}  // namespace presto
+
+extern "C" int presto_score_build_tree_noalloc(
+    const int32_t* topk_ids, const float* topk_logq, int B, int L, int k, int b,
+    const int32_t* ctx2, const presto_ngram3* ngram, float lambda, const float* lambda_d,
+    int policy, int beam_width, int N, int32_t* node_token, int32_t* node_parent,
+    int32_t* node_depth, float* node_score, int32_t* n_nodes, const int32_t* kv_len,
+    uint32_t* mask, int32_t* pos_ids, int32_t* dev_status, presto_stream_t stream) {
+  // the shape checks the plan needs; presto_score_build_tree_mask checks the rest
+  PRESTO_CHECK_ARG(B >= 1 && L >= 1 && k >= 1 && b >= 1 && b <= k && N >= 1 && beam_width >= 1);
+  PRESTO_CHECK_LIMIT(L <= kMaxL && k <= kMaxK && N <= kMaxN && beam_width <= kMaxN);
+  const BuildPlan pl = plan_build(L, k, b, N, beam_width, ngram != nullptr);
+  const size_t need = static_cast<size_t>(B) * (pl.ws_tables + pl.ws_p2);
+  if (need > kBuildStaticScratch) return PRESTO_ERR_UNSUPPORTED;
+  void* ws = build_static_scratch();
+  if (!ws) return PRESTO_ERR_CUDA;
+  return presto_score_build_tree_mask(topk_ids, topk_logq, B, L, k, b, ctx2, ngram, lambda,
+                                      lambda_d, policy, beam_width, N, node_token, node_parent,
+                                      node_depth, node_score, n_nodes, kv_len, mask, pos_ids, ws,
+                                      kBuildStaticScratch, dev_status, stream);
 }

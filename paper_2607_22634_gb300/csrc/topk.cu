@@ -53,8 +53,14 @@ template <>
 struct Elem<float> {
   static constexpr int kPerVec = 4;
   static constexpr int kBytes = 4;
+  static constexpr int kPairs = 2;
   static constexpr uint32_t kNegInfWord = 0xff800000u;
   __device__ static float load(const float* p) { return *p; }
+  // elements 2q and 2q + 1 of a vector
+  __device__ static float2 pair(const uint4& u, int q) {
+    return q == 0 ? make_float2(__uint_as_float(u.x), __uint_as_float(u.y))
+                  : make_float2(__uint_as_float(u.z), __uint_as_float(u.w));
+  }
   __device__ static float value(const uint4& u, int e) {
     return __uint_as_float(e == 0 ? u.x : e == 1 ? u.y : e == 2 ? u.z : u.w);
   }
@@ -81,8 +87,14 @@ template <>
 struct Elem<__nv_bfloat16> {
   static constexpr int kPerVec = 8;
   static constexpr int kBytes = 2;
+  static constexpr int kPairs = 4;
   static constexpr uint32_t kNegInfWord = 0xff80ff80u;
   __device__ static float load(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+  // elements 2q and 2q + 1 of a vector (the two halves of word q)
+  __device__ static float2 pair(const uint4& u, int q) {
+    const uint32_t w = q == 0 ? u.x : q == 1 ? u.y : q == 2 ? u.z : u.w;
+    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+  }
   __device__ static float value(const uint4& u, int e) {
     const uint32_t w = (e >> 1) == 0 ? u.x : (e >> 1) == 1 ? u.y : (e >> 1) == 2 ? u.z : u.w;
     return __uint_as_float((e & 1) ? (w & 0xffff0000u) : (w << 16));
@@ -381,30 +393,38 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
   const float m2 = mt * kLog2e;
   float st = 0.f, tt = 0.f;  // tt (ENT): Σ 2^u u
   if (mt != -INFINITY) {
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    // element e of a vector goes to accumulator e & 3, as pairs: packed float32x2
+    // FMA and add (each half rounds exactly as the scalar instruction)
+    const float2 l2 = make_float2(kLog2e, kLog2e), nm = make_float2(-m2, -m2);
+    float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
     if constexpr (!ENT) {
 #pragma unroll
       for (int i = 0; i < VMAX; ++i) {
 #pragma unroll
-        for (int e = 0; e < n; ++e) acc[e & 3] += ex2(fmaf(E::value(d[i], e), kLog2e, -m2));
+        for (int q = 0; q < E::kPairs; ++q) {
+          const float2 u = __ffma2_rn(E::pair(d[i], q), l2, nm);
+          acc[q & 1] = __fadd2_rn(acc[q & 1], make_float2(ex2(u.x), ex2(u.y)));
+        }
       }
-      st = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+      st = (acc[0].x + acc[0].y) + (acc[1].x + acc[1].y);
       if (xid >= 0) st += ex2(fmaf(xval, kLog2e, -m2));
     } else {
       // u is clamped at -256: 2^u flushes to 0 there, so -inf entries add 0 to both
-      float tac[4] = {0.f, 0.f, 0.f, 0.f};
+      float2 tac[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
       for (int i = 0; i < VMAX; ++i) {
 #pragma unroll
-        for (int e = 0; e < n; ++e) {
-          const float u = fmaxf(fmaf(E::value(d[i], e), kLog2e, -m2), -256.f);
-          const float p = ex2(u);
-          acc[e & 3] += p;
-          tac[e & 3] = fmaf(p, u, tac[e & 3]);
+        for (int q = 0; q < E::kPairs; ++q) {
+          float2 u = __ffma2_rn(E::pair(d[i], q), l2, nm);
+          u.x = fmaxf(u.x, -256.f);
+          u.y = fmaxf(u.y, -256.f);
+          const float2 p = make_float2(ex2(u.x), ex2(u.y));
+          acc[q & 1] = __fadd2_rn(acc[q & 1], p);
+          tac[q & 1] = __ffma2_rn(p, u, tac[q & 1]);
         }
       }
-      st = (acc[0] + acc[1]) + (acc[2] + acc[3]);
-      tt = (tac[0] + tac[1]) + (tac[2] + tac[3]);
+      st = (acc[0].x + acc[0].y) + (acc[1].x + acc[1].y);
+      tt = (tac[0].x + tac[0].y) + (tac[1].x + tac[1].y);
       if (xid >= 0) {
         const float u = fmaxf(fmaf(xval, kLog2e, -m2), -256.f);
         const float p = ex2(u);
@@ -559,21 +579,18 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
 
 // ---------------------------------------------------------------------------
 // Streaming variant, for problems of more than one wave of the kernel above (many
-// rows).  The CTA's span is cut into 4 KB chunks that the warps claim one at a time
-// from a counter in shared memory, so a warp whose copies land late takes fewer;
-// each warp's lane 0 keeps kWStages claimed chunks in flight as bulk copies into a
-// ring of the warp's own.  Each chunk's (max, Σ 2^u) pair is summed warp-wide in a
-// fixed order and kept under the chunk's index, and the CTA merges the pairs in chunk
-// order, so the result does not depend on which warp took which chunk.  Every warp
-// keeps its own top-k, sorted across lanes 0..k-1.  A candidate must reach theta: first
-// the k-th largest of all lanes' first-chunk maxima in the CTA (each a real
-// element), then the largest k-th value any warp of the CTA has published (a warp's
-// list holds k elements at or above its k-th value); nothing below theta is in the
-// row's top-k.  A lane whose chunk maximum is below theta costs one compare; a
-// candidate enters the warp's list by a warp-wide sorted insertion.  At the end
-// every warp sends the keys of its list at or above theta, and warp 0 the CTA's
-// (max, sum) pair, straight to the leader CTA of the row's cluster, which merges
-// them after one cluster barrier.
+// rows).  The CTA's span is cut into one contiguous piece per warp, and each warp
+// streams its piece in 4 KB chunks: its lane 0 keeps kWStages bulk copies in flight
+// in a ring of the warp's own.  Every lane keeps an online (max, Σ 2^u) pair and
+// every warp its own top-k, sorted across lanes 0..k-1.  A candidate must reach
+// theta: first the k-th largest of all lanes' first-chunk maxima in the CTA (each a
+// real element), then the largest k-th value any warp of the CTA has published (a
+// warp's list holds k elements at or above its k-th value); nothing below theta is
+// in the row's top-k.  A lane whose chunk maximum is below theta costs one compare;
+// a candidate enters the warp's list by a warp-wide sorted insertion.  When its
+// piece is done, every warp sends its (max, sum) pair and the keys of its list at or
+// above theta straight to the leader CTA of the row's cluster, which merges them,
+// in warp order, after one cluster barrier.
 // ---------------------------------------------------------------------------
 constexpr int kWThreads = 256;
 constexpr int kWWarps = kWThreads / 32;
@@ -583,24 +600,17 @@ constexpr int kWChunkBytes = kWChunkVec * 16;
 constexpr int kWStages = 3;
 constexpr size_t kWDynBytes = static_cast<size_t>(kWWarps) * kWStages * kWChunkBytes + 128;
 constexpr int kWCtasPerSm = 2;  // ~106 KB of shared memory and <= 128 registers a thread
-constexpr int kWSlots = kMaxParts * kWWarps;  // (part, warp) key lists gathered in the leader
-// chunks of one span at most (a float32 row of fewer than 2^18 elements), plus one
-// pair for the scalar head and tail elements
-constexpr int kWMaxChunks = ((kMaxV / 4) + kWChunkVec - 1) / kWChunkVec + 1;
-static_assert(kWStages == 3, "the claim queue below holds three chunks");
+constexpr int kWSlots = kMaxParts * kWWarps;  // (part, warp) results gathered in the leader
 
 struct WSmem {
   uint64_t full[kWWarps][kWStages];
   unsigned long long keys[kWSlots * kMaxK];  // leader: every warp's kept keys (0 = none)
   unsigned long long list[kMaxK];            // leader: the row's top-k, descending
-  float2 ms[kMaxParts];                      // leader: every part's (max log2, Σ 2^u)
-  float ts[kMaxParts];                       // leader, ENT: every part's Σ 2^u u
-  float2 cms[kWMaxChunks];                   // every chunk's (max log2, Σ 2^u)
-  float cts[kWMaxChunks];                    // ENT: every chunk's Σ 2^u u
+  float2 ms[kWSlots];                        // leader: every warp's (max log2, Σ 2^u)
+  float ts[kWSlots];                         // leader, ENT: every warp's Σ 2^u u
   uint32_t first[kWWarps * kMaxK];           // every warp's k largest first-chunk lane maxima
   float theta[kWWarps];                      // every warp's published k-th value
   float theta0;                              // the CTA's first threshold
-  int next;                                  // the next chunk of the span to claim
   int abort;                                 // set by any warp whose bounded wait ran out
 };
 
@@ -614,6 +624,21 @@ __device__ __forceinline__ unsigned long long warp_insert(unsigned long long& ls
   const unsigned long long up = __shfl_up_sync(kFull, lst, 1);
   if (lane < k) lst = lane == pos ? key : (lane > pos ? up : lst);
   return __shfl_sync(kFull, lst, k - 1);
+}
+
+// Move a lane's online (max, Σ 2^u[, Σ 2^u u]) pair to the maximum cm of new elements
+// when that is larger (u = x log2e - max2).
+template <bool ENT>
+__device__ __forceinline__ void rescale_to(float& mt, float& st, float& tt, float cm) {
+  if (cm > mt) {
+    if (mt != -INFINITY) {
+      const float dl = mt * kLog2e - cm * kLog2e;  // the old reference minus the new
+      const float f = ex2(dl);
+      if constexpr (ENT) tt = f * fmaf(dl, st, tt);
+      st *= f;
+    }
+    mt = cm;
+  }
 }
 
 // Merge pairs (m2_j, s_j[, t_j]) (log2-domain maxima, Σ 2^u, Σ 2^u u) held by the
@@ -660,10 +685,7 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
     sh.theta[warp] = -INFINITY;
     fence_barrier_init();
   }
-  if (tid == 0) {
-    sh.abort = 0;
-    sh.next = 0;
-  }
+  if (tid == 0) sh.abort = 0;
   __syncthreads();
   pdl_wait();  // the logits (and slot rows' accept results) come from earlier kernels
   const T* rowp = row_base<T>(a, row, part == 0 && tid == 0);
@@ -674,32 +696,24 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
   const uint4* vecp = reinterpret_cast<const uint4*>(rowp + head);
   const int v0 = min(nvec, part * a.vpt);  // vpt: vectors per span here
   const int v1 = min(nvec, v0 + a.vpt);
-  const int nch = (v1 - v0 + kWChunkVec - 1) / kWChunkVec;  // chunks of the span
+  const int per = (v1 - v0 + kWWarps - 1) / kWWarps;
+  const int wb = min(v1, v0 + warp * per);  // the warp's piece [wb, we)
+  const int we = min(v1, wb + per);
+  const int nch = (we - wb + kWChunkVec - 1) / kWChunkVec;  // chunks of the piece
   volatile int* abort = &sh.abort;
   volatile float* pub = sh.theta;
 
-  // claim the next chunk of the span and start its copy into ring slot s (lane 0);
-  // returns the chunk, >= nch when none is left
-  auto claim = [&](int s) -> int {
-    int c = nch;
-    if (lane == 0) {
-      c = atomicAdd(&sh.next, 1);
-      if (c < nch) {
-        const int vb = v0 + c * kWChunkVec;
-        const uint32_t bytes = static_cast<uint32_t>(min(kWChunkVec, v1 - vb)) * 16u;
-        mbar_arrive_expect_tx(&sh.full[warp][s], bytes);
-        bulk_g2s(ring + s * kWChunkBytes, vecp + vb, bytes, &sh.full[warp][s]);
-      }
-    }
-    return __shfl_sync(kFull, c, 0);
+  auto issue = [&](int c) {  // lane 0: chunk c of the piece into ring slot c % kWStages
+    const int st2 = c % kWStages;
+    const int vb = wb + c * kWChunkVec;
+    const uint32_t bytes = static_cast<uint32_t>(min(kWChunkVec, we - vb)) * 16u;
+    mbar_arrive_expect_tx(&sh.full[warp][st2], bytes);
+    bulk_g2s(ring + st2 * kWChunkBytes, vecp + vb, bytes, &sh.full[warp][st2]);
   };
-  // the warp's queue: chunks q0, q1, q2 are in flight in slots j, j + 1, j + 2
-  // (mod kWStages), j = chunks taken so far
-  int q0 = claim(0);
-  int q1 = claim(1);
-  int q2 = claim(2);
-  int j = 0;
+  if (lane == 0)
+    for (int c = 0; c < nch && c < kWStages; ++c) issue(c);
 
+  float mt = -INFINITY, st = 0.f, tt = 0.f;  // the lane's running max (plain), Σ 2^u, Σ 2^u u
   float theta = -INFINITY;                   // candidates: value >= theta ...
   unsigned long long thr = 0ull;             // ... and key > thr, the warp's k-th key
   unsigned long long lst = 0ull;             // lane j < k: the warp's j-th key
@@ -723,12 +737,11 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
       }
     }
   };
-  // the chunk at the head of the queue (q0 < nch): wait for its copy, take it into
-  // registers and refill its slot with a new claim; false (for the whole warp) when
-  // the wait gave up
-  auto take = [&](uint4 (&d)[kWVec], int& c) -> bool {
-    const int s = j % kWStages;
-    const bool ok = mbar_wait(&sh.full[warp][s], (j / kWStages) & 1, abort);
+  // chunk c: wait for its copy, take it into registers and refill its slot with
+  // chunk c + kWStages; false (for the whole warp) when the wait gave up
+  auto take = [&](uint4 (&d)[kWVec], int c) -> bool {
+    const int sg = c % kWStages;
+    const bool ok = mbar_wait(&sh.full[warp][sg], (c / kWStages) & 1, abort);
     if (!__all_sync(kFull, ok)) {
       if (lane == 0) {
         *abort = 1;
@@ -736,63 +749,65 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
       }
       return false;
     }
-    c = q0;
-    const int nv = min(kWChunkVec, v1 - (v0 + c * kWChunkVec));
+    const int nv = min(kWChunkVec, we - (wb + c * kWChunkVec));
     const uint32_t ni = E::kNegInfWord;
 #pragma unroll
     for (int i = 0; i < kWVec; ++i) {
       const int vi = i * 32 + lane;
-      d[i] = vi < nv ? *reinterpret_cast<const uint4*>(ring + s * kWChunkBytes + vi * 16)
+      d[i] = vi < nv ? *reinterpret_cast<const uint4*>(ring + sg * kWChunkBytes + vi * 16)
                      : make_uint4(ni, ni, ni, ni);
     }
     __syncwarp();
-    if (lane == 0) fence_proxy_async();  // the slot's reads come before its refill
-    const int qn = claim(s);
-    q0 = q1;
-    q1 = q2;
-    q2 = qn;
-    ++j;
+    if (lane == 0 && c + kWStages < nch) {  // the slot is free again: refill it
+      fence_proxy_async();
+      issue(c + kWStages);
+    }
     return true;
   };
-  // chunk c: the lane's maximum (returned), and the chunk's (max log2, Σ 2^u[, Σ 2^u u])
-  // summed over the warp in a fixed order into slot c; eight accumulators a lane
-  auto reduce = [&](const uint4 (&d)[kWVec], int c) -> float {
+  // the chunk's lane maximum (returned) and the lane's online (max, Σ 2^u) pair, log2
+  // domain; eight independent accumulators
+  auto reduce = [&](const uint4 (&d)[kWVec]) -> float {
     const float cm = E::template max_of<kWVec>(d);
-    const float mw = unordered(__reduce_max_sync(kFull, ordered(cm)));
-    float sc = 0.f, tc = 0.f;
-    if (mw != -INFINITY) {
-      const float m2 = mw * kLog2e;
-      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    rescale_to<ENT>(mt, st, tt, cm);
+    if (mt != -INFINITY) {
+      const float m2 = mt * kLog2e;
+      // element e of vector i goes to accumulator (i n + e) & 7, as pairs: packed
+      // float32x2 FMA and add (each half rounds exactly as the scalar instruction)
+      const float2 l2 = make_float2(kLog2e, kLog2e), nm = make_float2(-m2, -m2);
+      float2 acc[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) acc[j] = make_float2(0.f, 0.f);
       if constexpr (!ENT) {
 #pragma unroll
         for (int i = 0; i < kWVec; ++i)
 #pragma unroll
-          for (int e = 0; e < n; ++e)
-            acc[(i * n + e) & 7] += ex2(fmaf(E::value(d[i], e), kLog2e, -m2));
+          for (int q = 0; q < E::kPairs; ++q) {
+            const int j = (i * n / 2 + q) & 3;
+            const float2 u = __ffma2_rn(E::pair(d[i], q), l2, nm);
+            acc[j] = __fadd2_rn(acc[j], make_float2(ex2(u.x), ex2(u.y)));
+          }
       } else {
         // u clamped at -256: 2^u flushes to 0 there, so -inf adds 0 to both sums
-        float tac[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        float2 tac[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) tac[j] = make_float2(0.f, 0.f);
 #pragma unroll
         for (int i = 0; i < kWVec; ++i)
 #pragma unroll
-          for (int e = 0; e < n; ++e) {
-            const float u = fmaxf(fmaf(E::value(d[i], e), kLog2e, -m2), -256.f);
-            const float p = ex2(u);
-            acc[(i * n + e) & 7] += p;
-            tac[(i * n + e) & 7] = fmaf(p, u, tac[(i * n + e) & 7]);
+          for (int q = 0; q < E::kPairs; ++q) {
+            const int j = (i * n / 2 + q) & 3;
+            float2 u = __ffma2_rn(E::pair(d[i], q), l2, nm);
+            u.x = fmaxf(u.x, -256.f);
+            u.y = fmaxf(u.y, -256.f);
+            const float2 p = make_float2(ex2(u.x), ex2(u.y));
+            acc[j] = __fadd2_rn(acc[j], p);
+            tac[j] = __ffma2_rn(p, u, tac[j]);
           }
-        tc = ((tac[0] + tac[1]) + (tac[2] + tac[3])) + ((tac[4] + tac[5]) + (tac[6] + tac[7]));
+        tt += ((tac[0].x + tac[0].y) + (tac[1].x + tac[1].y)) +
+              ((tac[2].x + tac[2].y) + (tac[3].x + tac[3].y));
       }
-      sc = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      sc += __shfl_xor_sync(kFull, sc, off);
-      if constexpr (ENT) tc += __shfl_xor_sync(kFull, tc, off);
-    }
-    if (lane == 0) {
-      sh.cms[c] = make_float2(mw == -INFINITY ? -INFINITY : mw * kLog2e, sc);
-      if constexpr (ENT) sh.cts[c] = tc;
+      st += ((acc[0].x + acc[0].y) + (acc[1].x + acc[1].y)) +
+            ((acc[2].x + acc[2].y) + (acc[3].x + acc[3].y));
     }
     return cm;
   };
@@ -808,8 +823,8 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
   auto collect = [&](const uint4 (&d)[kWVec], float cm, int c) {
     const bool lane_hit = cm >= theta;
     if (!__any_sync(kFull, lane_hit)) return;
-    const int vb = v0 + c * kWChunkVec;
-    const int nv = min(kWChunkVec, v1 - vb);
+    const int vb = wb + c * kWChunkVec;
+    const int nv = min(kWChunkVec, we - vb);
     unsigned hits = 0u;
     if (lane_hit) {
 #pragma unroll
@@ -839,10 +854,11 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
   uint4 d[kWVec];
   bool alive = true;
   float cm0 = -INFINITY;
-  int c0 = -1;
-  if (q0 < nch) {
-    alive = take(d, c0);
-    if (alive) cm0 = reduce(d, c0);
+  int failed = -1;  // the chunk whose wait gave up
+  if (nch > 0) {
+    alive = take(d, 0);
+    if (alive) cm0 = reduce(d);
+    else failed = 0;
   }
   {
     uint32_t o = ordered(cm0);  // >= ordered(-inf) > 0: a taken lane's 0 never wins
@@ -876,78 +892,56 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
   theta = sh.theta0;
   if (lane == 0 && theta > pub[warp]) pub[warp] = theta;
 
-  // ---- the chunks
-  if (alive && c0 >= 0) collect(d, cm0, c0);
-  while (alive && q0 < nch) {
-    int c;
-    if (!take(d, c)) {
-      alive = false;
-      break;
-    }
-    const float cm = reduce(d, c);
-    refresh();
-    collect(d, cm, c);
-  }
-  if (!alive && lane == 0) {
-    // gave up: no copy of this warp may still be landing when the CTA exits
-    const int q[kWStages] = {q0, q1, q2};
-    for (int u = 0; u < kWStages; ++u)
-      if (q[u] < nch)
-        mbar_wait(&sh.full[warp][(j + u) % kWStages], ((j + u) / kWStages) & 1, nullptr);
-  }
-
   // ---- scalar elements (warp 0): the head of part 0 (lanes 0-6) and the tail of
-  // the last part (lanes 8-14), each < 8 elements; their pair goes to slot nch
+  // the last part (lanes 8-14), each < 8 elements, join the lanes' online pairs
   if (warp == 0) {
     int xid = -1;
     if (part == 0 && lane < head) xid = lane;
     if (part == a.parts - 1 && lane >= 8 && lane - 8 < V - tail0) xid = tail0 + (lane - 8);
     const float x = xid >= 0 ? E::load(rowp + xid) : -INFINITY;
-    float m2 = x * kLog2e, sx = 0.f, tx = 0.f;
-    if (xid >= 0 && x != -INFINITY) sx = 1.f;  // 2^(x log2e - m2) = 1, u = 0
-    else m2 = -INFINITY;
-    warp_merge_pairs<ENT>(m2, sx, tx);
-    if (lane == 0) {
-      sh.cms[nch] = make_float2(m2, sx);
-      if constexpr (ENT) sh.cts[nch] = tx;
+    rescale_to<ENT>(mt, st, tt, x);
+    if (xid >= 0 && mt != -INFINITY) {
+      const float u = fmaxf(fmaf(x, kLog2e, -mt * kLog2e), -256.f);
+      const float p = ex2(u);
+      st += p;
+      if constexpr (ENT) tt = fmaf(p, u, tt);
     }
-    refresh();
     unsigned m = (xid >= 0 && x >= theta) ? 1u : 0u;
     drain(m, [&](int) { return elem_key(x, xid); });
   }
 
-  // ---- every warp's keys at or above theta, and the CTA's (max, Σ) pair from its
-  // chunks' pairs in chunk order, into the leader
+  // ---- the chunks
+  if (alive && nch > 0) collect(d, cm0, 0);
+  for (int c = 1; alive && c < nch; ++c) {
+    if (!take(d, c)) {
+      alive = false;
+      failed = c;
+      break;
+    }
+    const float cm = reduce(d);
+    refresh();
+    collect(d, cm, c);
+  }
+  if (failed >= 0 && lane == 0) {
+    // gave up: no copy of this warp may still be landing when the CTA exits (chunks
+    // failed .. failed + kWStages - 1 were issued and not taken)
+    for (int c2 = failed; c2 < nch && c2 < failed + kWStages; ++c2)
+      mbar_wait(&sh.full[warp][c2 % kWStages], (c2 / kWStages) & 1, nullptr);
+  }
+
+  // ---- the warp's (max, Σ) pair and its keys at or above theta, into the leader
   refresh();
-  WSmem* ld = &sh;
-  if (a.parts > 1) ld = cg::this_cluster().map_shared_rank(&sh, 0);
-  if (lane < k)
-    ld->keys[(part * kWWarps + warp) * k + lane] =
-        (lst != 0ull && key_value(lst) >= theta) ? lst : 0ull;
-  __syncthreads();  // every chunk's pair is in place
-  if (warp == 0) {
-    // lane l folds pairs l, l + 32, ... in order; then the warp merges the lanes
-    float M = -INFINITY;
-    for (int c = lane; c <= nch; c += 32) M = fmaxf(M, sh.cms[c].x);
-    M = unordered(__reduce_max_sync(kFull, ordered(M)));
-    float sp = 0.f, tp = 0.f;
-    if (M != -INFINITY) {
-      for (int c = lane; c <= nch; c += 32) {
-        const float2 p = sh.cms[c];
-        if (p.x == -INFINITY) continue;
-        const float f = ex2(p.x - M);
-        sp = fmaf(p.y, f, sp);
-        if constexpr (ENT) tp = fmaf(f, fmaf(p.x - M, p.y, sh.cts[c]), tp);
-      }
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      sp += __shfl_xor_sync(kFull, sp, off);
-      if constexpr (ENT) tp += __shfl_xor_sync(kFull, tp, off);
-    }
+  {
+    float m2 = mt == -INFINITY ? -INFINITY : mt * kLog2e;
+    float sw = st, tw = tt;
+    warp_merge_pairs<ENT>(m2, sw, tw);
+    WSmem* ld = &sh;
+    if (a.parts > 1) ld = cg::this_cluster().map_shared_rank(&sh, 0);
+    const int slot = part * kWWarps + warp;
+    if (lane < k) ld->keys[slot * k + lane] = (lst != 0ull && key_value(lst) >= theta) ? lst : 0ull;
     if (lane == 0) {
-      ld->ms[part] = make_float2(M, sp);
-      if constexpr (ENT) ld->ts[part] = tp;
+      ld->ms[slot] = make_float2(m2, sw);
+      if constexpr (ENT) ld->ts[slot] = tw;
     }
   }
   if (a.parts > 1)
@@ -973,10 +967,24 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
   }
   float m_row = -INFINITY, s_row = 0.f, t_row = 0.f;
   if (warp == 0) {
-    m_row = lane < a.parts ? sh.ms[lane].x : -INFINITY;
-    s_row = lane < a.parts ? sh.ms[lane].y : 0.f;
-    if constexpr (ENT) t_row = lane < a.parts ? sh.ts[lane] : 0.f;
-    warp_merge_pairs<ENT>(m_row, s_row, t_row);
+    // lane l folds slots l and l + 32 (<= 64 slots), then the warp merges the lanes
+    const int P = a.parts * kWWarps;
+    float ma = lane < P ? sh.ms[lane].x : -INFINITY;
+    float sa = lane < P ? sh.ms[lane].y : 0.f;
+    float ta = 0.f;
+    if constexpr (ENT) ta = lane < P ? sh.ts[lane] : 0.f;
+    const float mb = lane + 32 < P ? sh.ms[lane + 32].x : -INFINITY;
+    const float sb = lane + 32 < P ? sh.ms[lane + 32].y : 0.f;
+    if constexpr (ENT) {
+      const float tb = lane + 32 < P ? sh.ts[lane + 32] : 0.f;
+      merge_mst(ma, sa, ta, mb, sb, tb);
+    } else {
+      merge_ms(ma, sa, mb, sb);
+    }
+    warp_merge_pairs<ENT>(ma, sa, ta);
+    m_row = ma;
+    s_row = sa;
+    t_row = ta;
   }
   __syncthreads();  // the row's list is complete
   if (warp == 0) write_row<ENT>(a, sh.list, row, m_row, s_row, t_row);

@@ -8,7 +8,7 @@
 //   * Every thread loads its whole share of the span (up to kMaxVpt 16-byte vectors)
 //     into registers with one burst of non-caching vector loads, then:
 //       - its maximum (packed bf16x2 max for bf16) and Σ exp(x - max) (one exp2 per
-//         element, four independent accumulators);
+//         element, four independent accumulators fed by packed float32x2 FMA/add);
 //       - the CTA's threshold tau = the k-th largest of the 16 warp maxima: at least
 //         k elements of the span are >= tau, so the span's top-k are among them;
 //       - the elements >= tau (vectors whose maximum is below tau are skipped) become
@@ -23,6 +23,8 @@
 //     s = Σ 2^u, u = x log2e - max2, each thread sums t = Σ 2^u u, and the merges
 //     carry t along (when the reference maximum drops by δ, t -> 2^δ (t + δ s)).
 //     Then H = ln s - ln2 t / s, and lambda_d = beta H / (H + C).
+//   * Problems of more rows than one wave of this kernel holds go to the streaming
+//     kernel further down (per-warp bulk-copy rings over longer spans).
 //   * With slot rows (self-speculative rounds, App. C (II)) row j of sequence b is
 //     read in place from slot slot_off + j of the deepest accepted node a*_b =
 //     accept_path[b][accept_len[b]], looked up on the device after the accept

@@ -100,23 +100,25 @@ def oracle_worker(args):
     inp = oracle_inputs(w)
     budget = args.cpu_seconds
     t0 = time.perf_counter()
-    oracle_step(w, inp)                           # warm-up round
+    for _ in range(max(1, args.warmup)):          # warm-up rounds, untimed
+        oracle_step(w, inp)
     first = time.perf_counter() - t0
     n, t_start = 0, time.perf_counter()
     while n < max(1, args.steps) and (n == 0 or time.perf_counter() - t_start < budget):
         oracle_step(w, inp)
         n += 1
     dt = time.perf_counter() - t_start
-    print(json.dumps({"rounds": n, "seconds": dt, "warmup_seconds": first}))
+    print(json.dumps({"rounds": n, "seconds": dt, "warmup_seconds": first,
+                      "warmup": max(1, args.warmup)}))
 
 
-def run_oracle(workload, seconds, max_steps):
+def run_oracle(workload, seconds, max_steps, warmup=1):
     env = dict(os.environ)
     for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "NUMEXPR_NUM_THREADS"):
         env[v] = "1"
     env["CUDA_VISIBLE_DEVICES"] = ""
     cmd = [sys.executable, os.path.abspath(__file__), "--oracle-worker", "--workload", workload,
-           "--cpu-seconds", str(seconds), "--steps", str(max_steps)]
+           "--cpu-seconds", str(seconds), "--steps", str(max_steps), "--warmup", str(warmup)]
     r = subprocess.run(cmd, capture_output=True, text=True, env=env)
     if r.returncode != 0:
         raise RuntimeError("oracle worker failed:\n" + r.stderr[-3000:])
@@ -130,13 +132,13 @@ def run_reference(args):
         return
     w = synth.WORKLOADS[args.workload]
     res = run_oracle(args.workload, seconds=min(60.0, max(10.0, 2.0 * args.steps)),
-                     max_steps=args.steps)
+                     max_steps=args.steps, warmup=args.warmup)
     value = res["rounds"] / res["seconds"]
     sample = (f"{res['rounds']} full oracle rounds of {args.steps} requested "
               f"(float64 numpy, one host thread): {workload_desc(w)}")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s",
-        "n_gpus": args.gpus, "steps": res["rounds"], "warmup": 1,
+        "n_gpus": args.gpus, "steps": res["rounds"], "warmup": res["warmup"],
         "ms_per_step": 1e3 / value, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": workload_desc(w), "parallelism": "replicas"},

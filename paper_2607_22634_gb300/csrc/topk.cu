@@ -628,6 +628,41 @@ __device__ __forceinline__ unsigned long long warp_insert(unsigned long long& ls
   return __shfl_sync(kFull, lst, k - 1);
 }
 
+// A warp's top-k state: lane j < k holds the j-th key in lst (0 = none), thr is the
+// k-th key (0 until k are held), theta the candidate threshold.
+struct WarpTop {
+  unsigned long long lst, thr;
+  float theta;
+};
+
+// The candidates of one vector (bit e of m: element e reaches theta, id0 + e its id),
+// one at a time through the warp's list; a raised theta is published to *pub_slot.
+// Out of line: the chunk loop's rare path, kept out of its instruction stream.  All
+// lanes of the warp call it.
+template <typename E>
+__device__ __noinline__ WarpTop drain_vector(WarpTop t, uint4 di, unsigned m, int id0, int k,
+                                             volatile float* pub_slot) {
+  const int lane = threadIdx.x & 31;
+  for (unsigned w = __ballot_sync(kFull, m != 0u); w; w = __ballot_sync(kFull, m != 0u)) {
+    const int src = __ffs(w) - 1;
+    const int e = __ffs(m) - 1;
+    const unsigned long long mine = m ? elem_key(E::value(di, e), id0 + e) : 0ull;
+    const unsigned long long key = __shfl_sync(kFull, mine, src);
+    if (lane == src) m &= m - 1u;
+    if (key > t.thr) {
+      t.thr = warp_insert(t.lst, key, k, lane);
+      if (t.thr) {
+        const float tv = key_value(t.thr);
+        if (tv > t.theta) {
+          t.theta = tv;
+          if (lane == 0) *pub_slot = tv;
+        }
+      }
+    }
+  }
+  return t;
+}
+
 // Move a lane's online (max, Σ 2^u[, Σ 2^u u]) pair to the maximum cm of new elements
 // when that is larger (u = x log2e - max2).
 template <bool ENT>
@@ -843,9 +878,11 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
         for (int e = 0; e < n; ++e)
           if (E::value(d[i], e) >= theta) m |= 1u << e;
       }
-      const int id0 = head + (vb + i * 32 + lane) * n;
-      const uint4 di = d[i];
-      drain(m, [&](int e) { return elem_key(E::value(di, e), id0 + e); });
+      const WarpTop t = drain_vector<E>(WarpTop{lst, thr, theta}, d[i], m,
+                                        head + (vb + i * 32 + lane) * n, k, &pub[warp]);
+      lst = t.lst;
+      thr = t.thr;
+      theta = t.theta;
     }
   };
 

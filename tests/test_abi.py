@@ -114,3 +114,25 @@ def test_trigram_key_packing():
     k = _lib.pack_trigram_keys([1, 262143], [2, 0], [3, 262143])
     assert int(k[0]) == (1 << 36) | (2 << 18) | 3
     assert int(k[1]) == (262143 << 36) | 262143
+
+
+def test_noalloc_build_host_checks():
+    """presto_score_build_tree_noalloc refuses, on the host and before any CUDA call,
+    shapes whose scratch exceeds its fixed 1 MiB array and malformed shapes; the
+    workspace query agrees on which shapes need more than the array holds."""
+    lib = P.load()
+    p = ctypes.c_void_p(16)  # never dereferenced: every call below is refused first
+    call = lambda B, L, k, b, Nn, W=1, lam=0.2, tbl=None: lib.presto_score_build_tree_noalloc(
+        p, p, B, L, k, b, p, tbl, ctypes.c_float(lam), N, 0 if W == 1 else 1, W, Nn,
+        p, p, p, p, p, N, N, N, N, N)
+    desc = ctypes.byref(_lib.Ngram3(16, 16, 20, -12.0))
+    # three N = 1024 trees (k = b = 8, with a table): ~1.18 MB of selection scratch
+    assert lib.presto_build_workspace_ex(3, 16, 8, 1024, 1) > (1 << 20)
+    assert call(3, 16, 8, 8, 1024, tbl=desc) == -2
+    # malformed shapes and limits
+    assert call(0, 16, 8, 8, 64) == -1
+    assert call(1, 16, 8, 9, 64) == -1        # b > k
+    assert call(1, 64, 8, 8, 64) == -2        # L above the limit
+    assert call(1, 16, 17, 8, 64) == -2       # k above the limit
+    assert call(1, 16, 8, 8, 1025) == -2      # N above the limit
+    assert call(1, 16, 8, 8, 64, W=0) == -1   # beam width 0

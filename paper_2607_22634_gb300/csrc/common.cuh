@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <mutex>
+
 #include "presto.h"
 
 #define PRESTO_CHECK_ARG(cond)                 \
@@ -35,6 +37,35 @@ __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a -
 
 // Per-device SM count, cached (host).
 int sm_count();
+
+constexpr int kMaxDevices = 64;
+
+// Kernel attributes (the dynamic shared-memory limit, permission for non-portable
+// cluster sizes) belong to the device that was current when they were set.  One
+// PerDeviceOnce per call site runs its setter once for each device the process
+// uses, with that device current, and returns the setter's outcome on every later
+// call on that device.
+class PerDeviceOnce {
+ public:
+  template <typename F>
+  cudaError_t run(F&& set) {
+    int dev = 0;
+    const cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(mu_);
+    if (!done_[dev]) {
+      res_[dev] = set();
+      done_[dev] = true;
+    }
+    return res_[dev];
+  }
+
+ private:
+  std::mutex mu_;
+  bool done_[kMaxDevices] = {};
+  cudaError_t res_[kMaxDevices] = {};
+};
 
 __device__ __forceinline__ void report(int32_t* st, int bits) {
   if (st) atomicOr(st, bits);

@@ -1141,10 +1141,13 @@ cudaError_t launch(const Plan& p, const Args& a, cudaStream_t stream) {
 
 template <typename T, bool ENT>
 cudaError_t launch_stream(const Plan& p, const Args& a, cudaStream_t stream) {
-  static const cudaError_t attr = cudaFuncSetAttribute(
-      topk_stream_kernel<T, ENT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-      static_cast<int>(kWDynBytes));
-  if (attr != cudaSuccess) return attr;
+  static PerDeviceOnce attr;
+  const cudaError_t ae = attr.run([] {
+    return cudaFuncSetAttribute(topk_stream_kernel<T, ENT>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                static_cast<int>(kWDynBytes));
+  });
+  if (ae != cudaSuccess) return ae;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(p.rows) * p.parts);
   cfg.blockDim = dim3(kWThreads);

@@ -733,13 +733,17 @@ Plan make_plan(int B, int N, int Hq, int Hkv, int Tmax, const int* active) {
   return p;
 }
 
+// The kernel's shared-memory limit and its permission for clusters of more than 8
+// CTAs, set once on every device that launches it.
 template <int D>
-void set_smem_attr() {
-  static std::once_flag once;
-  std::call_once(once, [] {
-    cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         Layout<D>::kAlloc);
-    cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+cudaError_t set_smem_attr() {
+  static PerDeviceOnce attr;
+  return attr.run([] {
+    cudaError_t e = cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         Layout<D>::kAlloc);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    return e;
   });
 }
 
@@ -755,7 +759,7 @@ const int* active_clusters() {
   std::lock_guard<std::mutex> lock(mu);
   int* act = cached[dev];
   if (done[dev]) return act;
-  set_smem_attr<D>();
+  if (set_smem_attr<D>() != cudaSuccess) cudaGetLastError();
   act[0] = 0;
   for (int c = 1; c <= kMaxSplits; ++c) {
     cudaLaunchConfig_t cfg{};
@@ -868,11 +872,11 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
   cfg.numAttrs = 2;
   cudaError_t err;
   if (D == 128) {
-    set_smem_attr<128>();
+    if (set_smem_attr<128>() != cudaSuccess) return PRESTO_ERR_CUDA;
     cfg.dynamicSmemBytes = Layout<128>::kAlloc;
     err = cudaLaunchKernelEx(&cfg, attn_kernel<128>, tq, tkc, tvc, tkt, tvt, a);
   } else {
-    set_smem_attr<64>();
+    if (set_smem_attr<64>() != cudaSuccess) return PRESTO_ERR_CUDA;
     cfg.dynamicSmemBytes = Layout<64>::kAlloc;
     err = cudaLaunchKernelEx(&cfg, attn_kernel<64>, tq, tkc, tvc, tkt, tvt, a);
   }

@@ -899,13 +899,15 @@ extern "C" int presto_score_build_tree_ex(const int32_t* topk_ids, const float* 
                                       ws, ws_bytes, dev_status, stream);
 }
 
-extern "C" int presto_score_build_tree_mask(
-    const int32_t* topk_ids, const float* topk_logq, int B, int L, int k, int b,
-    const int32_t* ctx2, const presto_ngram3* ngram, float lambda, const float* lambda_d,
-    int policy, int beam_width, int N, int32_t* node_token, int32_t* node_parent,
-    int32_t* node_depth, float* node_score, int32_t* n_nodes, const int32_t* kv_len,
-    uint32_t* mask, int32_t* pos_ids, void* ws, size_t ws_bytes, int32_t* dev_status,
-    presto_stream_t stream) {
+namespace presto {
+namespace {
+
+// Host-side checks of a tree-build call, run before any CUDA work.
+int build_arg_status(const int32_t* topk_ids, const float* topk_logq, int B, int L, int k, int b,
+                     const int32_t* ctx2, const presto_ngram3* ngram, float lambda, int policy,
+                     int beam_width, int N, const int32_t* node_token, const int32_t* node_parent,
+                     const int32_t* node_depth, const float* node_score, const int32_t* n_nodes,
+                     const int32_t* kv_len, const uint32_t* mask, const int32_t* pos_ids) {
   PRESTO_CHECK_ARG((kv_len && mask && pos_ids) || (!kv_len && !mask && !pos_ids));
   PRESTO_CHECK_ARG(topk_ids && topk_logq && ctx2 && node_token && node_parent && node_depth &&
                    node_score && n_nodes);
@@ -920,6 +922,23 @@ extern "C" int presto_score_build_tree_mask(
     PRESTO_CHECK_ARG(ngram->log2_cap >= 4 && ngram->log2_cap <= 30);
     PRESTO_CHECK_ARG(ngram->miss_logrho <= 0.f);
   }
+  return PRESTO_OK;
+}
+
+}  // namespace
+}  // namespace presto
+
+extern "C" int presto_score_build_tree_mask(
+    const int32_t* topk_ids, const float* topk_logq, int B, int L, int k, int b,
+    const int32_t* ctx2, const presto_ngram3* ngram, float lambda, const float* lambda_d,
+    int policy, int beam_width, int N, int32_t* node_token, int32_t* node_parent,
+    int32_t* node_depth, float* node_score, int32_t* n_nodes, const int32_t* kv_len,
+    uint32_t* mask, int32_t* pos_ids, void* ws, size_t ws_bytes, int32_t* dev_status,
+    presto_stream_t stream) {
+  const int arg_status = build_arg_status(topk_ids, topk_logq, B, L, k, b, ctx2, ngram, lambda,
+                                          policy, beam_width, N, node_token, node_parent,
+                                          node_depth, node_score, n_nodes, kv_len, mask, pos_ids);
+  if (arg_status != PRESTO_OK) return arg_status;
   Args a{};
   a.ids = topk_ids;
   a.logq = topk_logq;
@@ -963,12 +982,12 @@ extern "C" int presto_score_build_tree_mask(
   a.dev_status = dev_status;
   const size_t smem = pl.smem;
   if (smem > kDynSmemBudget) return PRESTO_ERR_UNSUPPORTED;
-  static bool attr_set = [] {
-    cudaFuncSetAttribute(build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         static_cast<int>(kDynSmemBudget));
-    return true;
-  }();
-  (void)attr_set;
+  static PerDeviceOnce smem_attr;
+  if (smem_attr.run([] {
+        return cudaFuncSetAttribute(build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    static_cast<int>(kDynSmemBudget));
+      }) != cudaSuccess)
+    return PRESTO_ERR_CUDA;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(B) * kCluster);
   cfg.blockDim = dim3(kThreads);
@@ -1037,9 +1056,11 @@ extern "C" int presto_score_build_tree_noalloc(
     int policy, int beam_width, int N, int32_t* node_token, int32_t* node_parent,
     int32_t* node_depth, float* node_score, int32_t* n_nodes, const int32_t* kv_len,
     uint32_t* mask, int32_t* pos_ids, int32_t* dev_status, presto_stream_t stream) {
-  // the shape checks the plan needs; presto_score_build_tree_mask checks the rest
-  PRESTO_CHECK_ARG(B >= 1 && L >= 1 && k >= 1 && b >= 1 && b <= k && N >= 1 && beam_width >= 1);
-  PRESTO_CHECK_LIMIT(L <= kMaxL && k <= kMaxK && N <= kMaxN && beam_width <= kMaxN);
+  // every host-side check first: a malformed call touches no CUDA state
+  const int arg_status = build_arg_status(topk_ids, topk_logq, B, L, k, b, ctx2, ngram, lambda,
+                                          policy, beam_width, N, node_token, node_parent,
+                                          node_depth, node_score, n_nodes, kv_len, mask, pos_ids);
+  if (arg_status != PRESTO_OK) return arg_status;
   const BuildPlan pl = plan_build(L, k, b, N, beam_width, ngram != nullptr);
   const size_t need = static_cast<size_t>(B) * (pl.ws_tables + pl.ws_p2);
   if (need > kBuildStaticScratch) return PRESTO_ERR_UNSUPPORTED;

@@ -163,10 +163,13 @@ extern "C" int presto_tree_mask(const int32_t* node_parent, const int32_t* node_
   const int threads = (N + 31) / 32 * 32;
   cudaLaunchConfig_t cfg{};
   const size_t rows_bytes = static_cast<size_t>(N) * (W + 1) * 4;
-  static const cudaError_t attr_ok = cudaFuncSetAttribute(
-      mask_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-      static_cast<int>(static_cast<size_t>(kMaxN) * (kMaxN / 32 + 1) * 4));
-  if (attr_ok != cudaSuccess) return PRESTO_ERR_CUDA;
+  static PerDeviceOnce smem_attr;
+  if (smem_attr.run([] {
+        return cudaFuncSetAttribute(
+            mask_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+            static_cast<int>(static_cast<size_t>(kMaxN) * (kMaxN / 32 + 1) * 4));
+      }) != cudaSuccess)
+    return PRESTO_ERR_CUDA;
   cfg.gridDim = dim3(static_cast<unsigned>(B));
   cfg.blockDim = dim3(static_cast<unsigned>(threads));
   cfg.dynamicSmemBytes = rows_bytes;

@@ -136,3 +136,17 @@ def test_noalloc_build_host_checks():
     assert call(1, 16, 17, 8, 64) == -2       # k above the limit
     assert call(1, 16, 8, 8, 1025) == -2      # N above the limit
     assert call(1, 16, 8, 8, 64, W=0) == -1   # beam width 0
+    # pointer, lambda, policy and table checks also run before the scratch lookup:
+    # here, with no GPU at all, each call still returns INVALID_ARG rather than a CUDA
+    # error
+    f = ctypes.c_float
+    full = lambda ids=p, lam=0.2, pol=0, tbl=None, kv=N, mk=N, po=N: \
+        lib.presto_score_build_tree_noalloc(ids, p, 1, 16, 8, 8, p, tbl, f(lam), N, pol, 1, 64,
+                                            p, p, p, p, p, kv, mk, po, N, N)
+    assert full(ids=N) == -1                  # null candidate ids
+    assert full(lam=-0.5) == -1               # negative lambda
+    assert full(lam=float("nan")) == -1
+    assert full(pol=3) == -1                  # unknown search policy
+    assert full(tbl=ctypes.byref(_lib.Ngram3(16, 16, 40, -12.0))) == -1  # table capacity
+    assert full(tbl=ctypes.byref(_lib.Ngram3(16, 16, 20, 0.5))) == -1    # miss log rho > 0
+    assert full(kv=p) == -1                   # kv_len without mask and pos_ids

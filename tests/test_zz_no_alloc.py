@@ -86,6 +86,12 @@ def test_noalloc_build_matches_workspace_entry_point(B, L, k, N, with_table, pol
     ref = P.presto_score_build_tree(ids, logq, ctx, ngram, lam, N, policy=policy, beam_width=W,
                                     kv_len=kv)
     torch.cuda.synchronize()
+    # an unrelated call (other seed and shape, the largest budget) first leaves the
+    # shared array full of its own data; then two checked calls in a row, each on the
+    # scratch the previous call left
+    oi, ol, oc, og = _inputs(B * 131 + 7, 1, 24, 10, True)
+    rc, _, st = _noalloc(oi, ol, oc, og, 0.3, 1024, P.SEARCH_BEST_FIRST, 1, to_dev([5]))
+    assert rc == 0 and st == 0
     for _ in range(2):  # two calls in a row share the one scratch array
         rc, got, st = _noalloc(ids, logq, ctx, ngram, lam, N, policy, W, kv)
         assert rc == 0 and st == 0

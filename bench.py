@@ -43,10 +43,18 @@ def parse_args(argv=None):
                    help="graph replays (each n_sets launches) of the per-call timing pass")
     p.add_argument("--e2e-steps", type=int, default=2000)
     p.add_argument("--cpu-seconds", type=float, default=15.0)
+    p.add_argument("--repeats", type=int, default=5,
+                   help="timed regions of --steps rounds each (at least)")
+    p.add_argument("--repeat-seconds", type=float, default=1.0,
+                   help="keep repeating the timed region for at least this long")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-variants", action="store_true",
                    help="skip timing the search policies, adaptive lambda and slot top-k")
     p.add_argument("--oracle-worker", action="store_true", help=argparse.SUPPRESS)
+    p.add_argument("--oracle-mode", choices=["round", "mp", "subset", "check"], default="round",
+                   help=argparse.SUPPRESS)
+    p.add_argument("--check-in", default=None, help=argparse.SUPPRESS)
+    p.add_argument("--parity-out", default=None, help=argparse.SUPPRESS)
     return p.parse_args(argv)
 
 
@@ -57,93 +65,289 @@ def workload_desc(w):
 
 
 # ---------------------------------------------------------------- CPU oracle
+# The oracle runs only here: in the cpu_baseline leg of the GPU arm and in the
+# reference arm, always in a subprocess that sees no GPU.
 
-def oracle_step(w, inp):
-    """One full draft-and-verify round with the CPU oracle (float64)."""
-    from oracle import presto_oracle as O
-    ids, logq, _ = O.topk_logsoftmax(inp["logits"], w.k)
-    ids = ids.reshape(w.B, w.L, w.k)
-    logq = logq.reshape(w.B, w.L, w.k)
-    tree = O.best_first_tree(ids, logq, inp["ctx"], inp["table"], w.miss_logrho, w.lam,
-                             w.branching, w.N, "fp32")
-    mask, _ = O.tree_mask(tree["parent"], tree["depth"], tree["n_nodes"], inp["kv_len"], w.N)
-    for lay in inp["layers"]:
-        O.tree_attention(lay["q"], lay["k_cache"], lay["v_cache"], inp["kv_len"], lay["k_tree"],
-                         lay["v_tree"], mask, tree["n_nodes"])
-    O.accept(tree["token"], tree["parent"], tree["n_nodes"], inp["target"], w.L)
+# workloads whose attention the oracle times on a subset of (sequence, kv head)
+# pairs, scaled to the whole round by flops
+ATTN_SUBSET = {"batched_ragged": ([0, 1], [0]), "long_ctx": ([0], [0])}
 
 
-def oracle_inputs(w):
+def oracle_inputs(w, attn_f64=True):
+    """Set 0 of the workload (the GPU arm's input set 0) for the oracle: logits,
+    context, table, the tree's target tokens, one attention layer (float64, or
+    float32 arrays the oracle converts slice by slice when attn_f64 is False)."""
     import numpy as np
     import synth
     from oracle import presto_oracle as O
     logits = synth.drafter_logits(w)
     a, b, t, lr = synth.trigram_entries(w)
     att = synth.attention_inputs(w, device="cpu")
-    f64 = lambda x: x.double().numpy()
+    conv = (lambda x: x.double().numpy()) if attn_f64 else (lambda x: x.float().numpy())
     ids, logq, _ = O.topk_logsoftmax(logits.reshape(w.rows, w.V).double().numpy(), w.k)
     table = O.make_table(a, b, t, lr) if w.use_table else None
     ctx = synth.ctx_tokens(w).numpy()
     tree = O.best_first_tree(ids.reshape(w.B, w.L, w.k), logq.reshape(w.B, w.L, w.k), ctx, table,
                              w.miss_logrho, w.lam, w.branching, w.N, "fp32")
     target = synth.target_tokens(w, logits, tree["token"], tree["parent"], tree["n_nodes"]).numpy()
-    layer = {k: f64(v) for k, v in att.items() if k != "kv_len"}
+    layer = {k: conv(v) for k, v in att.items() if k != "kv_len"}
+    layer["q"] = att["q"].double().numpy()
     return {"logits": logits.reshape(w.rows, w.V).double().numpy(), "ctx": ctx, "table": table,
-            "kv_len": att["kv_len"].numpy(), "layers": [layer] * w.layers, "target": target,
+            "kv_len": att["kv_len"].numpy(), "layer": layer, "target": target,
             "n_entries": int(np.size(a))}
 
 
+def oracle_round(w, inp, seqs=None, kv_heads=None, clock=None, n_layers=None):
+    """One draft-and-verify round with the CPU oracle (float64; the tree search in
+    float32, as the kernels take its decisions).  Attention runs on every layer (or
+    n_layers of them), or on the (seqs, kv_heads) subset of each.  `clock`
+    (optional dict) collects the seconds of each step."""
+    import time as _t
+    from oracle import presto_oracle as O
+    t0 = _t.perf_counter()
+    ids, logq, lse = O.topk_logsoftmax(inp["logits"], w.k)
+    t1 = _t.perf_counter()
+    ids3, logq3 = ids.reshape(w.B, w.L, w.k), logq.reshape(w.B, w.L, w.k)
+    tree = O.best_first_tree(ids3, logq3, inp["ctx"], inp["table"], w.miss_logrho, w.lam,
+                             w.branching, w.N, "fp32")
+    mask, pos = O.tree_mask(tree["parent"], tree["depth"], tree["n_nodes"], inp["kv_len"], w.N)
+    t2 = _t.perf_counter()
+    lay = inp["layer"]
+    out = None
+    for _ in range(w.layers if n_layers is None else n_layers):
+        out, _ = O.tree_attention(lay["q"], lay["k_cache"], lay["v_cache"], inp["kv_len"],
+                                  lay["k_tree"], lay["v_tree"], mask, tree["n_nodes"],
+                                  seqs=seqs, kv_heads=kv_heads)
+    t3 = _t.perf_counter()
+    acc, path, bonus = O.accept(tree["token"], tree["parent"], tree["n_nodes"], inp["target"], w.L)
+    t4 = _t.perf_counter()
+    if clock is not None:
+        for key, dt in (("topk", t1 - t0), ("build_mask", t2 - t1), ("attention", t3 - t2),
+                        ("accept", t4 - t3)):
+            clock[key] = clock.get(key, 0.0) + dt
+    return {"ids": ids, "logq": logq, "lse": lse, "token": tree["token"],
+            "parent": tree["parent"], "depth": tree["depth"], "score": tree["score"],
+            "n_nodes": tree["n_nodes"], "mask": mask, "pos": pos, "attn": out,
+            "accept_len": acc, "accept_path": path, "bonus": bonus}
+
+
+def attention_flops(w, kv_len, n_nodes, mask, seqs=None, kv_heads=None):
+    """4 Hq' D sum_b sum_i (T_b + |anc(i)|) over the sequences and kv heads given
+    (all by default), Hq' = the query heads of those kv heads; one layer."""
+    import numpy as np
+    G = w.Hq // w.Hkv
+    heads = (w.Hkv if kv_heads is None else len(kv_heads)) * G
+    total = 0
+    for b in (range(w.B) if seqs is None else seqs):
+        n = int(n_nodes[b])
+        anc = int(np.unpackbits(np.asarray(mask[b, :n], np.uint32).view(np.uint8)).sum())
+        total += int(kv_len[b]) * n + anc
+    return 4.0 * heads * w.D * total
+
+
+# -- multi-process oracle: one process per host core, each holding the inputs
+_MP = {}
+
+
+def _mp_init(workload):
+    import synth
+    w = synth.WORKLOADS[workload]
+    _MP["w"] = w
+    _MP["inp"] = oracle_inputs(w)
+
+
+def _mp_topk(rows):
+    from oracle import presto_oracle as O
+    return O.topk_logsoftmax(_MP["inp"]["logits"][rows[0]:rows[1]], _MP["w"].k)
+
+
+def _mp_tree(args):
+    from oracle import presto_oracle as O
+    w, inp = _MP["w"], _MP["inp"]
+    b, ids_b, logq_b = args
+    return O.best_first_tree(ids_b, logq_b, inp["ctx"][b:b + 1], inp["table"], w.miss_logrho,
+                             w.lam, w.branching, w.N, "fp32")
+
+
+def _mp_attn(args):
+    from oracle import presto_oracle as O
+    w, inp = _MP["w"], _MP["inp"]
+    b, g, mask, n_nodes = args
+    lay = inp["layer"]
+    G = w.Hq // w.Hkv
+    out, _ = O.tree_attention(lay["q"], lay["k_cache"], lay["v_cache"], inp["kv_len"],
+                              lay["k_tree"], lay["v_tree"], mask, n_nodes, seqs=[b], kv_heads=[g])
+    return out[b, :, g * G:(g + 1) * G]
+
+
+def oracle_round_mp(w, inp, pool, procs):
+    """oracle_round with its independent pieces spread over a process pool: top-k
+    rows, one tree per sequence, attention per (sequence, kv head); the mask and
+    the acceptance (microseconds) stay in the parent."""
+    import numpy as np
+    from oracle import presto_oracle as O
+    R = w.rows
+    cuts = [(R * i // procs, R * (i + 1) // procs) for i in range(procs)]
+    parts = pool.map(_mp_topk, [c for c in cuts if c[1] > c[0]])
+    ids = np.concatenate([p[0] for p in parts]).reshape(w.B, w.L, w.k)
+    logq = np.concatenate([p[1] for p in parts]).reshape(w.B, w.L, w.k)
+    trees = pool.map(_mp_tree, [(b, ids[b:b + 1], logq[b:b + 1]) for b in range(w.B)])
+    tree = {key: np.concatenate([t[key] for t in trees]) for key in trees[0]}
+    mask, _ = O.tree_mask(tree["parent"], tree["depth"], tree["n_nodes"], inp["kv_len"], w.N)
+    for _ in range(w.layers):
+        pool.map(_mp_attn, [(b, g, mask, tree["n_nodes"]) for b in range(w.B)
+                            for g in range(w.Hkv)])
+    O.accept(tree["token"], tree["parent"], tree["n_nodes"], inp["target"], w.L)
+
+
 def oracle_worker(args):
-    """Runs in a fresh single-threaded process: time full oracle rounds."""
+    """Runs in a fresh process with one BLAS thread and no GPU.  Modes:
+    round  full rounds on one thread (and, with --parity-out, input set 0's round
+           results saved for the GPU arm to compare with);
+    mp     full rounds with one process per host core;
+    subset the round's steps on one thread, attention on ATTN_SUBSET's pairs,
+           scaled to the whole round (all layers) by flops."""
     import synth
     w = synth.WORKLOADS[args.workload]
-    inp = oracle_inputs(w)
     budget = args.cpu_seconds
+    mode = args.oracle_mode
+    if mode == "check":
+        print(json.dumps(oracle_check(w, args.check_in)))
+        return
+    if mode == "subset":
+        seqs, heads = ATTN_SUBSET[args.workload]
+        inp = oracle_inputs(w, attn_f64=False)
+        clock = {}
+        res = oracle_round(w, inp, seqs=seqs, kv_heads=heads, clock=clock, n_layers=1)
+        full = attention_flops(w, inp["kv_len"], res["n_nodes"], res["mask"]) * w.layers
+        sub = attention_flops(w, inp["kv_len"], res["n_nodes"], res["mask"], seqs, heads)
+        attn_s = clock["attention"] * full / sub
+        secs = clock["topk"] + clock["build_mask"] + attn_s + clock["accept"]
+        print(json.dumps({"seconds_per_round": secs, "steps": clock,
+                          "attention_scaled_seconds": attn_s, "attention_scale": full / sub,
+                          "subset": {"seqs": seqs, "kv_heads": heads}}))
+        return
+    inp = oracle_inputs(w)
+    pool, procs = None, 1
+    if mode == "mp":
+        import multiprocessing as mp
+        procs = max(1, os.cpu_count() or 1)
+        pool = mp.get_context("spawn").Pool(procs, initializer=_mp_init, initargs=(args.workload,))
+        step = lambda: oracle_round_mp(w, inp, pool, procs)
+    else:
+        step = lambda: oracle_round(w, inp)
     t0 = time.perf_counter()
     for _ in range(max(1, args.warmup)):          # warm-up rounds, untimed
-        oracle_step(w, inp)
+        step()
     first = time.perf_counter() - t0
     n, t_start = 0, time.perf_counter()
     while n < max(1, args.steps) and (n == 0 or time.perf_counter() - t_start < budget):
-        oracle_step(w, inp)
+        step()
         n += 1
     dt = time.perf_counter() - t_start
+    if pool is not None:
+        pool.close()
+        pool.join()
+    if args.parity_out:
+        import numpy as np
+        np.savez(args.parity_out, **oracle_round(w, inp))
     print(json.dumps({"rounds": n, "seconds": dt, "warmup_seconds": first,
-                      "warmup": max(1, args.warmup)}))
+                      "warmup": max(1, args.warmup), "procs": procs}))
 
 
-def run_oracle(workload, seconds, max_steps, warmup=1):
+def oracle_check(w, gpu_file):
+    """Each step of the GPU's round on input set 0 against the oracle applied to that
+    step's inputs as the GPU had them (so floating-point near-ties upstream cannot
+    make later steps differ): the tree from the GPU's candidates, the mask and
+    position ids from the GPU's tree, attention with the GPU's mask, acceptance on
+    the GPU's tree with its target tokens.  Exact, except scores (1e-5 relative) and
+    attention (2e-2 max abs)."""
+    import numpy as np
+    import synth
+    from oracle import presto_oracle as O
+    g = dict(np.load(gpu_file))
+    g["mask"] = np.ascontiguousarray(g["mask"]).view(np.uint32)  # 32-bit words, unsigned
+    a, b, t, lr = synth.trigram_entries(w)
+    table = O.make_table(a, b, t, lr) if w.use_table else None
+    ctx = synth.ctx_tokens(w).numpy()
+    ids = g["ids"].astype(np.int64).reshape(w.B, w.L, w.k)
+    logq = g["logq"].astype(np.float64).reshape(w.B, w.L, w.k)
+    tree = O.best_first_tree(ids, logq, ctx, table, w.miss_logrho, w.lam, w.branching, w.N, "fp32")
+    c = {}
+    c["tree"] = bool(all(np.array_equal(tree[k], g[k]) for k in ("token", "parent", "depth",
+                                                                  "n_nodes")))
+    c["tree_scores_equal"] = bool(np.array_equal(np.asarray(tree["score"], np.float32),
+                                                 g["score"].astype(np.float32)))
+    mask, pos = O.tree_mask(g["parent"], g["depth"], g["n_nodes"], g["kv_len"], w.N)
+    c["mask"] = bool(np.array_equal(mask, g["mask"]))
+    if not c["mask"]:
+        bad = np.argwhere((mask != g["mask"]).any(axis=2))
+        b0, i0 = (int(bad[0][0]), int(bad[0][1])) if len(bad) else (0, 0)
+        c["mask_rows_differ"] = int(len(bad))
+        c["mask_first_diff"] = {"seq": b0, "node": i0, "gpu": g["mask"][b0, i0].tolist(),
+                                "oracle": mask[b0, i0].tolist(),
+                                "shapes": [list(mask.shape), list(g["mask"].shape)]}
+    c["pos_ids"] = bool(np.array_equal(pos, g["pos_ids"]))
+    if w.layers == 1:
+        att = synth.attention_inputs(w, device="cpu")
+        f64 = lambda x: x.double().numpy()
+        out, _ = O.tree_attention(f64(att["q"]), f64(att["k_cache"]), f64(att["v_cache"]),
+                                  g["kv_len"], f64(att["k_tree"]), f64(att["v_tree"]),
+                                  g["mask"], g["n_nodes"])
+        c["attention_max_abs"] = float(np.abs(out - g["attn"]).max())
+    else:
+        c["attention_max_abs"] = None  # the GPU output is the last layer's; checked in tests
+    acc, path, bonus = O.accept(g["token"], g["parent"], g["n_nodes"], g["target"], w.L)
+    c["accept"] = bool(np.array_equal(acc, g["accept_len"]) and np.array_equal(path, g["accept_path"])
+                       and np.array_equal(bonus, g["bonus"]))
+    return c
+
+
+def run_oracle(workload, seconds, max_steps, warmup=1, mode="round", parity_out=None,
+               check_in=None):
     env = dict(os.environ)
     for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "NUMEXPR_NUM_THREADS"):
         env[v] = "1"
     env["CUDA_VISIBLE_DEVICES"] = ""
     cmd = [sys.executable, os.path.abspath(__file__), "--oracle-worker", "--workload", workload,
-           "--cpu-seconds", str(seconds), "--steps", str(max_steps), "--warmup", str(warmup)]
+           "--cpu-seconds", str(seconds), "--steps", str(max_steps), "--warmup", str(warmup),
+           "--oracle-mode", mode]
+    if parity_out:
+        cmd += ["--parity-out", parity_out]
+    if check_in:
+        cmd += ["--check-in", check_in]
     r = subprocess.run(cmd, capture_output=True, text=True, env=env)
     if r.returncode != 0:
         raise RuntimeError("oracle worker failed:\n" + r.stderr[-3000:])
     return json.loads(r.stdout.strip().splitlines()[-1])
 
 
+def bench_config(w, world):
+    """The `config` both arms print (so the driver sees the same workload)."""
+    return {"workload": workload_desc(w), "parallelism": "replicas" if world > 1 else "1 GPU"}
+
+
 def run_reference(args):
     import synth
     rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
     if rank != 0:
         return
     w = synth.WORKLOADS[args.workload]
     res = run_oracle(args.workload, seconds=min(60.0, max(10.0, 2.0 * args.steps)),
-                     max_steps=args.steps, warmup=args.warmup)
+                     max_steps=args.steps, warmup=args.warmup, mode="mp")
     value = res["rounds"] / res["seconds"]
-    sample = (f"{res['rounds']} full oracle rounds of {args.steps} requested "
-              f"(float64 numpy, one host thread): {workload_desc(w)}")
+    sample = (f"{res['rounds']} full oracle rounds of {args.steps} requested (float64 numpy; "
+              f"top-k rows, trees and attention (sequence, kv head) pairs spread over "
+              f"{res['procs']} processes, one per host core): {workload_desc(w)}")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s",
         "n_gpus": args.gpus, "steps": res["rounds"], "warmup": res["warmup"],
         "ms_per_step": 1e3 / value, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": workload_desc(w), "parallelism": "replicas"},
-        "cpu_baseline": {"value": value, "unit": "steps/s", "cores": 1, "kind": "oracle",
-                         "sample": sample},
+        "config": bench_config(w, world),
+        "cpu_baseline": {"value": value, "unit": "steps/s", "cores": res["procs"],
+                         "host_cores": os.cpu_count(), "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }), flush=True)
@@ -344,6 +548,111 @@ def time_variants(args, P, w, step, sets, side, ngram):
     return out
 
 
+def cpu_baseline(args, w):
+    """The oracle timed on the host cores, each leg in a subprocess without a GPU:
+    one thread (full rounds of the workload's input set 0, whose results come back
+    in a temporary file), one process per host core (full rounds), and for the two
+    large workloads one round on a subset of (sequence, kv head) pairs, scaled to
+    the whole round by attention flops.  Returns (cpu_baseline dict, results file)."""
+    import tempfile
+    host = os.cpu_count()
+    fd, path = tempfile.mkstemp(suffix=".npz")
+    os.close(fd)
+    out = {"value": None, "unit": "steps/s", "cores": None, "host_cores": host, "kind": "oracle",
+           "sample": None}
+    try:
+        r1 = run_oracle(args.workload, args.cpu_seconds, 10 ** 6, mode="round", parity_out=path)
+        one = {"value": r1["rounds"] / r1["seconds"], "unit": "steps/s", "cores": 1,
+               "sample": f"{r1['rounds']} full oracle rounds ({r1['seconds']:.1f} s), one thread"}
+        out["single_thread"] = one
+        out.update(value=one["value"], cores=1, sample=one["sample"])
+    except Exception as e:  # reported, not fatal
+        out["sample"] = f"failed: {e}"[:300]
+        os.unlink(path)
+        return out, None
+    try:
+        r2 = run_oracle(args.workload, args.cpu_seconds, 10 ** 6, mode="mp")
+        out.update(value=r2["rounds"] / r2["seconds"], cores=r2["procs"],
+                   sample=(f"{r2['rounds']} full oracle rounds ({r2['seconds']:.1f} s) of the "
+                           f"same workload (input set 0), numpy float64, with top-k rows, "
+                           f"trees and attention (sequence, kv head) pairs spread over "
+                           f"{r2['procs']} processes, one per host core"))
+    except Exception as e:
+        out["multi_process"] = f"failed: {e}"[:300]
+    by = {}
+    for name in ATTN_SUBSET:
+        try:
+            r = run_oracle(name, 0, 1, mode="subset")
+            by[name] = {"seconds_per_round": r["seconds_per_round"],
+                        "steps_per_s": 1.0 / r["seconds_per_round"], "cores": 1,
+                        "step_seconds": r["steps"],
+                        "sample": (f"one round on one thread: top-k, tree, mask and accept in "
+                                   f"full; attention of sequences {r['subset']['seqs']} x kv "
+                                   f"heads {r['subset']['kv_heads']} of one layer, scaled by "
+                                   f"attention flops (x{r['attention_scale']:.1f}) to every "
+                                   f"sequence, head and layer")}
+        except Exception as e:
+            by[name] = {"failed": f"{e}"[:300]}
+    out["by_workload"] = by
+    return out, path
+
+
+def round_parity(w, step, st0, graph0, oracle_file):
+    """Replays the round on input set 0 (the graph the timed region replays) and checks
+    it against the oracle: the top-k against the oracle's top-k of the same logits
+    (ids exact; log q and lse within 1e-5 relative), then every later step against
+    the oracle applied to that step's inputs as the GPU had them (oracle_check).  The
+    tree of the oracle's own chain may differ where float32 near-ties decide a node;
+    `chain_tree_equal` reports whether it did."""
+    import tempfile
+    import numpy as np
+    import torch
+    o = dict(np.load(oracle_file))
+    step.dev_status.zero_()
+    if graph0 is not None:
+        graph0.replay()
+    else:
+        step.run(st0["logits"], st0["ctx"], st0["layers"], st0["kv_len"], st0["target"])
+    torch.cuda.synchronize()
+    h = lambda t: t.cpu().numpy()
+
+    def rel(a, b):
+        a, b = np.asarray(a, np.float64), np.asarray(b, np.float64)
+        both = np.isinf(a) & np.isinf(b) & (np.sign(a) == np.sign(b))
+        e = np.where(both, 0.0, np.abs(a - b) / np.maximum(1.0, np.abs(b)))
+        return float(e.max()) if e.size else 0.0
+
+    R = w.rows
+    g = {"ids": h(step.topk_ids).reshape(R, w.k), "logq": h(step.topk_logq).reshape(R, w.k),
+         "mask": h(step.mask).view(np.uint32), "pos_ids": h(step.pos_ids),
+         "attn": h(step.attn_out.float()).astype(np.float64), "accept_len": h(step.accept_len),
+         "accept_path": h(step.accept_path), "bonus": h(step.bonus), "target": h(st0["target"]),
+         "kv_len": h(st0["kv_len"])}
+    g.update({k: h(v) for k, v in step.tree.items()})
+    c = {"topk_ids": bool(np.array_equal(g["ids"], o["ids"])),
+         "logq_rel_err": rel(g["logq"], o["logq"]),
+         "lse_rel_err": rel(h(step.lse).reshape(R), o["lse"]),
+         "chain_tree_equal": bool(all(np.array_equal(g[k], o[k]) for k in ("token", "parent",
+                                                                          "depth", "n_nodes"))),
+         "dev_status": int(step.dev_status.item())}
+    fd, path = tempfile.mkstemp(suffix=".npz")
+    os.close(fd)
+    try:
+        np.savez(path, **g)
+        c.update(run_oracle(w.name, 0, 1, mode="check", check_in=path))
+    except Exception as e:  # reported
+        c["check_failed"] = f"{e}"[:300]
+    finally:
+        os.unlink(path)
+    ok = (c["topk_ids"] and c["logq_rel_err"] <= 1e-5 and c["lse_rel_err"] <= 1e-5
+          and c.get("tree", False) and c.get("tree_scores_equal", False) and c.get("mask", False)
+          and c.get("pos_ids", False) and c.get("accept", False) and c["dev_status"] == 0
+          and (c.get("attention_max_abs") is None or c["attention_max_abs"] <= 2e-2))
+    return {"ok": ok, "input_set": 0, "checks": c,
+            "against": ("the CPU oracle: top-k from the same logits; every later step from "
+                        "that step's inputs as the GPU had them")}
+
+
 def max_over_ranks(x, device=None):
     """The largest of every rank's x (the job's time is its slowest replica's); x
     itself on a single process."""
@@ -362,7 +671,7 @@ def job_throughput(world, steps_per_rank, seconds):
     return world * steps_per_rank / seconds
 
 
-def time_workload_rooflines(args, P, hbm, tc):
+def time_workload_rooflines(args, P, hbm, tc, tc_sus):
     """Top-k and one attention layer of the larger workloads, each timed the way the
     per-call numbers are (a graph of launches over inputs that together exceed L2),
     against the measured peaks: the kernels' rooflines where the work is large enough
@@ -415,6 +724,7 @@ def time_workload_rooflines(args, P, hbm, tc):
             "attention_layer_us": attn_us,
             "attention_tflops": flops / (attn_us * 1e-6) / 1e12,
             "attention_tensor_frac": flops / (attn_us * 1e-6) / 1e12 / tc,
+            "attention_tensor_frac_sustained": flops / (attn_us * 1e-6) / 1e12 / tc_sus,
             "attention_hbm_frac": abytes / (attn_us * 1e-6) / 1e9 / hbm,
         }
         del att, mask
@@ -608,24 +918,39 @@ def run_ours(args):
         chain.replay()
     torch.cuda.synchronize()
 
-    # ---- timed region
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
+    # ---- timed region: K rounds, repeated (each repeat between its own pair of CUDA
+    # events on the launch stream) at least --repeats times and for at least
+    # --repeat-seconds, so that the clock sampler sees the load; value = the median
+    # repeat (max over ranks), with its spread
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
+    evs = []
     with ClockSampler(gpu_smi_id(dev)) as clk:
         t_wall0 = time.time()
-        e0.record(stream)
-        timed_rounds()
-        e1.record(stream)
+        while len(evs) < max(1, args.repeats) or (time.time() - t_wall0 < args.repeat_seconds
+                                                  and len(evs) < 5000):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            timed_rounds()
+            e1.record(stream)
+            evs.append((e0, e1))
+            if len(evs) % 64 == 0:
+                e1.synchronize()
         torch.cuda.synchronize()
         t_wall1 = time.time()
     if world > 1:
         dist.barrier()
-    ms = max_over_ranks(e0.elapsed_time(e1), dev)
+    rep_ms = [a.elapsed_time(b) for a, b in evs]
+    ms = max_over_ranks(statistics.median(rep_ms), dev)
     clocks = clk.summary(t_wall0, t_wall1)
     value = job_throughput(world, args.steps, ms / 1e3)
+    repeats = {"n": len(rep_ms), "ms_per_step_median": ms / args.steps,
+               "ms_per_step_min": min(rep_ms) / args.steps,
+               "ms_per_step_max": max(rep_ms) / args.steps,
+               "value_min": job_throughput(world, args.steps, max(rep_ms) / 1e3),
+               "value_max": job_throughput(world, args.steps, min(rep_ms) / 1e3)}
 
     # ---- per-call durations: each call alone, captured n_sets times in a row
     # (rotating over the input sets, so the big inputs come from HBM) into a CUDA
@@ -668,67 +993,47 @@ def run_ours(args):
 
     # ---- end to end through the public API with host buffers: every round's inputs
     # (logits, context, target tokens, each layer's q and tree K/V; the KV cache is
-    # resident) sit packed in one pinned host buffer and go to the device in one copy,
-    # into a staging buffer the round reads; the round's results come back in one copy
-    names = ["logits", "ctx", "target"] + [f"{k}{j}" for j in range(w.layers)
-                                          for k in ("q", "k_tree", "v_tree")]
-
+    # resident) sit packed in one pinned host buffer and go to the device in one copy;
+    # the round's results come back in one copy that the host waits for.  StagedRounds
+    # double-buffers the staging, so round i + 1's copy in overlaps round i's compute
     def tensors_of(st):
         out = [st["logits"], st["ctx"], st["target"]]
         for lay in st["layers"]:
             out += [lay["q"], lay["k_tree"], lay["v_tree"]]
         return out
 
-    offs, pos = [], 0
-    for t in tensors_of(sets[0]):
-        offs.append(pos)
-        pos += -(-t.numel() * t.element_size() // 256) * 256
-    staging = torch.empty(pos, dtype=torch.uint8, device=dev)
+    def bind(v):
+        layers_s = [{"q": v[3 + 3 * j], "k_tree": v[4 + 3 * j], "v_tree": v[5 + 3 * j],
+                     "k_cache": sets[0]["layers"][j]["k_cache"],
+                     "v_cache": sets[0]["layers"][j]["v_cache"]} for j in range(w.layers)]
+        return v[0], v[1], layers_s, sets[0]["kv_len"], v[2]
 
-    def views(buf):
-        return [buf[o:o + t.numel() * t.element_size()].view(t.dtype).view(t.shape)
-                for o, t in zip(offs, tensors_of(sets[0]))]
-
-    host = []
-    for st in sets:
-        hb = torch.empty(pos, dtype=torch.uint8).pin_memory()
-        for v, t in zip(views(hb), tensors_of(st)):
-            v.copy_(t.cpu())
-        host.append(hb)
-    sv = dict(zip(names, views(staging)))
-    layers_s = [{"q": sv[f"q{j}"], "k_tree": sv[f"k_tree{j}"], "v_tree": sv[f"v_tree{j}"],
-                 "k_cache": sets[0]["layers"][j]["k_cache"], "v_cache": sets[0]["layers"][j]["v_cache"]}
-                for j in range(w.layers)]
-    staging.copy_(host[0])
-    g_staged = (step.capture(sv["logits"], sv["ctx"], layers_s, sets[0]["kv_len"], sv["target"])
-                if use_graph else None)
-    res_host = torch.empty(step.result.numel(), dtype=torch.int32).pin_memory()
-    h2d = pos
-    d2h = res_host.numel() * res_host.element_size()
-
-    def e2e_step(i):
-        staging.copy_(host[i % n_sets], non_blocking=True)
-        if g_staged is not None:
-            g_staged.replay()
-        else:
-            step.run(sv["logits"], sv["ctx"], layers_s, sets[0]["kv_len"], sv["target"])
-        res_host.copy_(step.result, non_blocking=True)
-        stream.synchronize()                      # the host reads the accepted length
-
-    for i in range(min(20, args.e2e_steps)):
-        e2e_step(i)
+    staged = P.StagedRounds(step, tensors_of(sets[0]), bind)
+    host = [staged.pack(tensors_of(st)) for st in sets]
+    h2d = staged.nbytes
+    d2h = step.result.numel() * step.result.element_size()
+    n_warm = min(20, args.e2e_steps)
+    staged.start(host[0])
+    for i in range(n_warm):
+        staged.run(i, host[(i + 1) % n_sets])
     n_e2e = args.e2e_steps
     t0 = time.perf_counter()
-    for i in range(n_e2e):
-        e2e_step(i)
+    for i in range(n_warm, n_warm + n_e2e):
+        staged.run(i, host[(i + 1) % n_sets])
     e2e_s = max_over_ranks(time.perf_counter() - t0, dev)
     e2e_value = job_throughput(world, n_e2e, e2e_s)
+    torch.cuda.synchronize()
 
-    # ---- roofline of the dominant call
+    # ---- roofline of the dominant call (attention work from input set 0's tree)
     peaks, peak_src = load_peaks()
+    if use_graph:
+        graphs[0].replay()
+    else:
+        one(0)
+    torch.cuda.synchronize()
     tree = {k: v.cpu().numpy() for k, v in step.tree.items()}
     mask = step.mask.cpu().numpy().view(np.uint32)
-    kv = sets[0]["kv_len"].cpu().numpy()  # the last rounds ran the staged graph (set 0 state)
+    kv = sets[0]["kv_len"].cpu().numpy()
     anc = sum(int(np.unpackbits(mask[b, : int(tree["n_nodes"][b])].view(np.uint8)).sum())
               for b in range(w.B))
     n_used = int(tree["n_nodes"].sum())
@@ -739,7 +1044,10 @@ def run_ours(args):
     topk_bytes = w.B * w.L * w.V * esz
     dominant = max(us, key=us.get)
     hbm = float(peaks["hbm_gbs"])
-    tc = float(peaks.get("bf16_tflops_sustained", peaks["bf16_tflops"]))
+    # each call is timed alone (a graph of that call's launches), so a contraction's
+    # fraction is taken of the burst tensor peak; the sustained one is reported too
+    tc = float(peaks["bf16_tflops"])
+    tc_sus = float(peaks.get("bf16_tflops_sustained", tc))
     if dominant == "attention":
         t_us = us["attention"]
         t_tensor = attn_flops / (tc * 1e12) * 1e6
@@ -753,6 +1061,7 @@ def run_ours(args):
         roof["kernel"] = "presto_tree_attention (attn_kernel)"
         roof["traffic"] = profiled_traffic("attention")
         roof["tensor_frac"] = attn_flops / (t_us * 1e-6) / 1e12 / tc
+        roof["tensor_frac_sustained"] = attn_flops / (t_us * 1e-6) / 1e12 / tc_sus
         roof["hbm_frac"] = attn_bytes / (t_us * 1e-6) / 1e9 / hbm
         roof["algorithmic"] = {"flops": attn_flops, "bytes": attn_bytes}
     else:
@@ -767,7 +1076,10 @@ def run_ours(args):
                     "kernel": dominant, "traffic": None}
     if roof.get("achieved") is not None:
         roof["frac"] = roof["achieved"] / roof["peak"]
-    roof["peak_source"] = f"{peak_src} ({'sustained' if roof.get('unit') == 'TFLOP/s' else 'copy'})"
+    roof["peak_source"] = (f"{peak_src} ({'bf16 burst; tensor_frac of burst, tensor_frac_sustained'
+                           f' of sustained' if roof.get('unit') == 'TFLOP/s' else 'copy'}); "
+                           f"attention tensor_frac of burst {tc}, tensor_frac_sustained of "
+                           f"sustained {tc_sus} TFLOP/s")
     roof["duration_us"] = t_us
     roof["timing"] = (f"CUDA events around {args.kernel_steps} replays of a graph of {n_sets} "
                       f"launches of the call alone (one per input set); per launch")
@@ -775,20 +1087,18 @@ def run_ours(args):
 
     by_workload = None
     if not args.no_variants:
-        by_workload = time_workload_rooflines(args, P, hbm, tc)
+        by_workload = time_workload_rooflines(args, P, hbm, tc, tc_sus)
         by_workload["long_ctx_full_depth"] = time_full_depth(args, P)
 
-    cpu = None
+    # ---- the CPU oracle on the host cores (rank 0, one GPU): one thread, one process
+    # per core, and the large workloads on a subset scaled by flops; the one-thread
+    # leg also returns input set 0's round, which the GPU round is checked against
+    cpu, parity = None, None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        try:
-            r = run_oracle(args.workload, args.cpu_seconds, 10 ** 6)
-            cpu = {"value": r["rounds"] / r["seconds"], "unit": "steps/s", "cores": 1,
-                   "kind": "oracle",
-                   "sample": f"{r['rounds']} full oracle rounds ({r['seconds']:.1f} s) of the "
-                             f"same workload on input set 0, numpy float64, one host thread"}
-        except Exception as e:  # reported, not fatal
-            cpu = {"value": None, "unit": "steps/s", "cores": 1, "kind": "oracle",
-                   "sample": f"failed: {e}"[:300]}
+        cpu, oracle_file = cpu_baseline(args, w)
+        if oracle_file is not None:
+            parity = round_parity(w, step, sets[0], graphs[0] if use_graph else None, oracle_file)
+            os.unlink(oracle_file)
 
     if rank == 0:
         print(json.dumps({
@@ -796,13 +1106,14 @@ def run_ours(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": workload_desc(w),
-                       "inputs": f"{n_sets} rotating input sets of {set_bytes / 1e6:.1f} MB "
+            "config": bench_config(w, world),
+            "timing": {"inputs": f"{n_sets} rotating input sets of {set_bytes / 1e6:.1f} MB "
                                  f"({n_sets * set_bytes / 1e6:.0f} MB > 2 x L2), no L2 flush",
                        "cuda_graph": (f"timed rounds replay graphs of {n_sets} rounds (the input "
                                       f"sets in turn); e2e one graph per round") if use_graph
                                      else False,
-                       "parallelism": "replicas" if world > 1 else "1 GPU"},
+                       "repeats": repeats},
+            "parity": parity,
             "roofline": roof,
             "topk_hbm_frac": topk_frac,
             "call_us": us,
@@ -812,9 +1123,10 @@ def run_ours(args):
             "e2e": {"value": e2e_value, "unit": "steps/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h,
                     "note": "every round: its inputs (logits, q, tree K/V, ctx, targets) packed "
-                            "in one pinned host buffer, one copy in; the round; accept_len/"
-                            "path/bonus in one copy out; a host synchronisation. KV cache "
-                            "resident"},
+                            "in one pinned host buffer, one copy in (on a copy stream, into one "
+                            "of two staging buffers, overlapping the previous round); the "
+                            "round (a CUDA graph); accept_len/path/bonus in one copy out; a "
+                            "host wait for it. KV cache resident (StagedRounds)"},
             "clocks": clocks,
             "gpu_launches": args.steps * step.kernels_per_round(w.layers),
         }), flush=True)

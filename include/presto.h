@@ -84,6 +84,17 @@ const char* presto_status_string(int status);
 int presto_version(void);
 
 /*
+ * presto_selftest_wait_timeout - a diagnostic with no counterpart in the paper: it
+ * exercises the bounded in-kernel waits.  One GPU thread waits up to wait_cycles SM
+ * cycles (0 <= wait_cycles <= about 2e9, the library's own limit, roughly a
+ * second) for a barrier phase that nothing completes; the wait runs out, ORs
+ * PRESTO_DEV_TIMEOUT into *dev_status (device int32, required) and the kernel
+ * returns normally, leaving the context usable.  Enqueued on `stream`.
+ */
+int presto_selftest_wait_timeout(int32_t* dev_status, long long wait_cycles,
+                                 presto_stream_t stream);
+
+/*
  * presto_topk - per-row log-softmax and top-k (the drafter's position-wise
  * marginals q_d of §2.3, Eq. marginal-surrogate; "extracts top-k diffusion
  * candidates", §4.3; k = 10 in §5.1).

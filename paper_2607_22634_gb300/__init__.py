@@ -22,6 +22,7 @@ from ._lib import (  # noqa: F401
     presto_build_workspace,
     presto_score_build_tree,
     presto_score_build_tree_noalloc,
+    presto_selftest_wait_timeout,
     presto_topk,
     presto_topk_entropy,
     presto_topk_slots,
@@ -29,4 +30,4 @@ from ._lib import (  # noqa: F401
     presto_tree_attention,
     presto_tree_mask,
 )
-from .step import DraftVerifyStep  # noqa: F401
+from .step import DraftVerifyStep, StagedRounds  # noqa: F401

@@ -72,6 +72,7 @@ _SIGS = {
     "presto_tree_attention": (_I, [_P, _P, _P, _P, _I, _P, _P, _P, _P, _I, _I, _I, _I, _I,
                                    ctypes.c_float, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "presto_accept": (_I, [_P, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P]),
+    "presto_selftest_wait_timeout": (_I, [_P, ctypes.c_longlong, _P]),
 }
 
 _lib = None
@@ -445,3 +446,11 @@ def presto_accept(node_token, node_parent, node_depth, mask, n_nodes, target_tok
                               _ptr(accept_path), _ptr(bonus), _ptr(dev_status), _stream(stream))
     _check(st, "presto_accept")
     return accept_len, accept_path, bonus
+
+
+def presto_selftest_wait_timeout(dev_status, wait_cycles, stream=None):
+    """One GPU thread waits wait_cycles SM cycles for a barrier phase nothing
+    completes; PRESTO_DEV_TIMEOUT is ORed into dev_status (a device int32 tensor)."""
+    _need(dev_status, torch.int32, (1,), "dev_status")
+    _check(load().presto_selftest_wait_timeout(_ptr(dev_status), int(wait_cycles), _stream(stream)),
+           "presto_selftest_wait_timeout")

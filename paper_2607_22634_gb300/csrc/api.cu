@@ -4,6 +4,19 @@
 #include "common.cuh"
 
 namespace presto {
+namespace {
+
+// One thread waits, with a limit of `limit` SM cycles, for a phase of an mbarrier
+// that nothing ever arrives on; the wait runs out and reports PRESTO_DEV_TIMEOUT
+// exactly as the kernels' own waits do.  Nothing asynchronous is in flight.
+__global__ void wait_selftest_kernel(int32_t* dev_status, long long limit) {
+  __shared__ uint64_t bar;
+  mbar_init(&bar, 1);
+  fence_barrier_init();
+  if (!mbar_wait(&bar, 0, nullptr, limit)) report(dev_status, PRESTO_DEV_TIMEOUT);
+}
+
+}  // namespace
 
 int sm_count() {
   static int counts[64] = {0};
@@ -38,3 +51,11 @@ extern "C" const char* presto_status_string(int status) {
 }
 
 extern "C" int presto_version(void) { return (1 << 16) | 0; }
+
+extern "C" int presto_selftest_wait_timeout(int32_t* dev_status, long long wait_cycles,
+                                            presto_stream_t stream) {
+  PRESTO_CHECK_ARG(dev_status);
+  PRESTO_CHECK_ARG(wait_cycles >= 0 && wait_cycles <= presto::kWaitCycles);
+  presto::wait_selftest_kernel<<<1, 1, 0, stream>>>(dev_status, wait_cycles);
+  return presto::launch_status();
+}

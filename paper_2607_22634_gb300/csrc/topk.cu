@@ -33,6 +33,7 @@
 
 #include <cooperative_groups.h>
 
+#include <algorithm>
 #include <cmath>
 #include <mutex>
 
@@ -45,6 +46,7 @@ constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMaxParts = 8;     // spans of a row = CTAs of its (portable) cluster
 constexpr int kCandCap = 1024;   // candidate keys per CTA and round
+constexpr size_t kPrefetchCap = 48ull << 20;  // bytes a streaming launch asks L2 to prefetch
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr unsigned kFull = 0xffffffffu;
 static_assert(kWarps >= kMaxK, "tau needs at least k warp maxima");
@@ -193,6 +195,7 @@ struct Args {
   const void* logits;
   long long row_stride;  // elements
   int V, k, parts, vpt;
+  uint32_t pf_bytes;  // streaming kernel: L2 prefetch budget of each warp (bytes)
   int32_t* topk_ids;
   float* topk_logq;
   float* lse;
@@ -377,6 +380,14 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
   int xid = -1;
   if (part == 0 && tid < head) xid = tid;
   if (part == a.parts - 1 && tid >= 8 && tid - 8 < V - tail0) xid = tail0 + (tid - 8);
+  // before the dependency wait, ask L2 for the span (slot rows are only known after
+  // it): a hint that reads nothing into the SM, so it cannot return data older than
+  // the loads below, and its DRAM latency overlaps the previous kernel
+  if (!a.acc_len && tid < kWarps && v1 > v0) {
+    const int per = (v1 - v0 + kWarps - 1) / kWarps;
+    const int b = v0 + tid * per, e = min(v1, b + per);
+    if (e > b) prefetch_l2_bulk(vecp + b, static_cast<uint32_t>(e - b) * 16u);
+  }
 
   pdl_wait();  // the logits may come from the previous kernel on the stream
   uint4 d[VMAX];
@@ -724,18 +735,35 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
   }
   if (tid == 0) sh.abort = 0;
   __syncthreads();
+  // the warp's piece [wb, we) of the row's aligned vectors
+  auto geometry = [&](const T* rp, int& head, int& tail0, const uint4*& vecp, int& wb, int& we) {
+    const int mis = static_cast<int>(reinterpret_cast<uintptr_t>(rp) & 15);
+    head = min(V, mis == 0 ? 0 : (16 - mis) / eb);
+    const int nvec = (V - head) / n;
+    tail0 = head + nvec * n;
+    vecp = reinterpret_cast<const uint4*>(rp + head);
+    const int v0 = min(nvec, part * a.vpt);  // vpt: vectors per span here
+    const int v1 = min(nvec, v0 + a.vpt);
+    const int per = (v1 - v0 + kWWarps - 1) / kWWarps;
+    wb = min(v1, v0 + warp * per);
+    we = min(v1, wb + per);
+  };
+  // before the dependency wait (plain rows only; slot rows are known after it), ask
+  // L2 for the head of the warp's piece: a hint that reads nothing into the SM, so
+  // it cannot return data older than the copies below
+  if (!a.acc_len && lane == 0 && a.pf_bytes > 0) {
+    int h0, t0, b0, e0;
+    const uint4* vp;
+    geometry(row_base<T>(a, row, false), h0, t0, vp, b0, e0);
+    const uint32_t bytes = min(a.pf_bytes, static_cast<uint32_t>(max(0, e0 - b0)) * 16u);
+    for (uint32_t o = 0; o < bytes; o += 65536u)
+      prefetch_l2_bulk(reinterpret_cast<const char*>(vp + b0) + o, min(65536u, bytes - o));
+  }
   pdl_wait();  // the logits (and slot rows' accept results) come from earlier kernels
   const T* rowp = row_base<T>(a, row, part == 0 && tid == 0);
-  const int mis = static_cast<int>(reinterpret_cast<uintptr_t>(rowp) & 15);
-  const int head = min(V, mis == 0 ? 0 : (16 - mis) / eb);
-  const int nvec = (V - head) / n;
-  const int tail0 = head + nvec * n;
-  const uint4* vecp = reinterpret_cast<const uint4*>(rowp + head);
-  const int v0 = min(nvec, part * a.vpt);  // vpt: vectors per span here
-  const int v1 = min(nvec, v0 + a.vpt);
-  const int per = (v1 - v0 + kWWarps - 1) / kWWarps;
-  const int wb = min(v1, v0 + warp * per);  // the warp's piece [wb, we)
-  const int we = min(v1, wb + per);
+  int head, tail0, wb, we;
+  const uint4* vecp;
+  geometry(rowp, head, tail0, vecp, wb, we);
   const int nch = (we - wb + kWChunkVec - 1) / kWChunkVec;  // chunks of the piece
   volatile int* abort = &sh.abort;
   volatile float* pub = sh.theta;
@@ -1210,6 +1238,13 @@ int topk_common(const void* logits, int dtype, int B, int L, int V, long long ro
   a.k = k;
   a.parts = p.parts;
   a.vpt = p.vpt;
+  if (p.stream && !slots) {
+    // the whole problem up to kPrefetchCap bytes, the head of every warp's piece beyond
+    const size_t total = static_cast<size_t>(B) * L * V * eb;
+    const size_t warps = static_cast<size_t>(p.rows) * p.parts * kWWarps;
+    const size_t per = total <= kPrefetchCap ? total : kPrefetchCap / warps;
+    a.pf_bytes = static_cast<uint32_t>(std::min<size_t>(per, 0x7fffffffu) / 16 * 16);
+  }
   a.topk_ids = topk_ids;
   a.topk_logq = topk_logq;
   a.lse = lse;

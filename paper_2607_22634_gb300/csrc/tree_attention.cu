@@ -30,7 +30,8 @@
 //     either way), the cluster synchronises (release / acquire), and each CTA
 //     merges a slice of the rows over the splits with log-sum-exp weights, all loads
 //     of a row issued together.
-// Every wait is bounded; on time-out the CTA records PRESTO_DEV_TIMEOUT and unwinds.
+// Every wait is bounded; on time-out the CTA records PRESTO_DEV_TIMEOUT, lets its
+// copies and MMAs in flight complete (bounded), then frees its TMEM and exits.
 #include <cuda_bf16.h>
 
 #include <cooperative_groups.h>
@@ -67,6 +68,8 @@ constexpr int kWidePartialKeys = 1024;  // prefixes shorter than this merge floa
 constexpr int kMaxSplits = 16;  // KV splits of a row block = CTAs of its cluster
 
 struct Args {
+  const __nv_bfloat16* k_cache;  // [B, Hkv, Tmax, D] (for the L2 prefetch)
+  const __nv_bfloat16* v_cache;
   const int32_t* kv_len;
   const uint32_t* mask;
   const int32_t* n_nodes;
@@ -104,6 +107,7 @@ struct Bars {
   uint64_t k_full[kMaxStages], k_empty[kMaxStages];
   uint64_t v_full[kMaxStages], v_empty[kMaxStages];
   uint64_t s_full[2], p_full[2], o_done[2];
+  uint64_t drain;  // after a timed-out wait: every MMA issued so far has completed
 };
 
 // Packed fp32 pairs (f32x2 arithmetic issues one instruction per two values) and
@@ -187,6 +191,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars.p_full[t], kSoftThreads);
       mbar_init(&bars.o_done[t], 1);
     }
+    mbar_init(&bars.drain, 1);
     abort_flag = 0;
     fence_barrier_init();
   }
@@ -197,6 +202,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // before the dependency wait, ask L2 for this split's KV-prefix rows: no kernel of
+  // the round writes the KV cache, and a prefetch is a hint that reads nothing into
+  // the SM, so its DRAM traffic overlaps the previous kernels whatever they write.
+  // The split's range is taken from kv_len as read now and the node budget N (the
+  // exact split below uses the node count the build writes): a stale read only
+  // misplaces the hint by a tile.
+  if (tid == 0) {
+    const int kvh = min(max(*reinterpret_cast<const volatile int32_t*>(a.kv_len + b), 0), a.Tmax);
+    const int pt = (kvh + kBN - 1) / kBN;
+    const int tot = pt + (a.N + kBN - 1) / kBN;
+    const int per_h = (tot + a.n_splits - 1) / a.n_splits;
+    const int tb = min(split * per_h, pt);
+    const int te = min(tb + per_h, pt);
+    if (te > tb) {
+      const size_t row0 = (static_cast<size_t>(b) * a.Hkv + g) * a.Tmax;
+      const int t0 = tb * kBN, t1 = min(te * kBN, kvh);
+      const uint32_t bytes = static_cast<uint32_t>(t1 - t0) * D * 2u;
+      prefetch_l2_bulk(a.k_cache + (row0 + t0) * D, bytes);
+      prefetch_l2_bulk(a.v_cache + (row0 + t0) * D, bytes);
+    }
+  }
   pdl_wait();  // the mask and node counts come from the previous kernels on the stream
   const int kv_raw = a.kv_len[b];
   const int nn_raw = a.n_nodes[b];
@@ -230,6 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     report(a.dev_status, PRESTO_DEV_TIMEOUT);
   };
 
+  int issued = 0;  // K or V tiles this warp's lane 0 has issued (the loaders)
   if (nt > 0 && warp == kKWarp) {
     // ------------------------------------------------------------ Q and K loads
     if (lane == 0) {
@@ -258,6 +285,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_3d(dst + p * Ly::kKVPanel, &tm_kt, p * 64, g,
                         b * a.N + (tree0 + j - n_prefix) * kBN, &bars.k_full[st]);
         }
+        issued = j + 1;
       }
     }
   } else if (nt > 0 && warp == kVWarp) {
@@ -282,6 +310,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_3d(dst + p * Ly::kKVPanel, &tm_vt, p * 64, g,
                         b * a.N + (tree0 + j - n_prefix) * kBN, &bars.v_full[st]);
         }
+        issued = j + 1;
       }
     }
   } else if (nt > 0 && warp == kMmaWarp) {
@@ -521,6 +550,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (node < a.N && a.lse)
         a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] =
             used ? (m + log2f(l)) * kLn2 : -INFINITY;
+    }
+  }
+
+  // ---- unwind after a timed-out wait.  Before the TMEM is freed and the CTA exits,
+  // nothing asynchronous may still target them: each loader waits (bounded) for the
+  // last copy it issued into every stage (and for Q), whether or not anyone consumed
+  // it, and the MMA warp commits to the drain barrier, which completes once every
+  // MMA it issued has.  A drain wait that gives up too means the GPU no longer
+  // answers; the status word already holds PRESTO_DEV_TIMEOUT.
+  if (__syncthreads_or(*abort)) {
+    if (nt > 0 && (warp == kKWarp || warp == kVWarp) && lane == 0) {
+      uint64_t* full = warp == kKWarp ? bars.k_full : bars.v_full;
+      const int S = warp == kKWarp ? Ly::kKStages : Ly::kVStages;
+      if (warp == kKWarp) mbar_wait(&bars.q_full, 0, nullptr);
+      for (int j = max(0, issued - S); j < issued; ++j) mbar_wait(&full[j % S], (j / S) & 1, nullptr);
+    }
+    if (nt > 0 && warp == kMmaWarp) {
+      mma_commit_warp(&bars.drain);
+      mbar_wait(&bars.drain, 0, nullptr);
     }
   }
 
@@ -840,6 +888,8 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
             make_map(&tvt, v_tree, Du, Hkv, static_cast<uint64_t>(B) * N, Du * e, Du * Hkv * e, 1,
                      kBN);
   if (!ok) return PRESTO_ERR_CUDA;
+  a.k_cache = static_cast<const __nv_bfloat16*>(k_cache);
+  a.v_cache = static_cast<const __nv_bfloat16*>(v_cache);
   a.kv_len = kv_len;
   a.mask = mask;
   a.n_nodes = n_nodes;

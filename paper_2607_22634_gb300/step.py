@@ -124,3 +124,78 @@ class DraftVerifyStep:
         with torch.cuda.graph(g, stream=s):
             self.run(logits, ctx2, layers, kv_len, target_token, stream=s)
         return g
+
+
+class StagedRounds:
+    """Rounds fed from pinned host memory, with each round's input copy overlapped
+    with the previous round's compute.
+
+    One round's inputs (the tensors of `example`, e.g. logits, context, target
+    tokens and each layer's q and tree K/V; the KV cache stays resident) are packed
+    into one contiguous 256-byte-aligned layout.  Two device staging buffers hold
+    that layout, and one CUDA graph of the round is captured per buffer.  `run(i)`
+    runs round i from its staging buffer while a copy stream brings round i + 1's
+    inputs into the other buffer, then copies round i's results (accept_len, path
+    and bonus, one contiguous buffer) to pinned host memory and waits for them:
+    every round still moves its own inputs in and its results out.
+
+    `bind(views)` maps the staged tensors (a list of device views, in the order of
+    `example`) to the arguments of DraftVerifyStep.run:
+    (logits, ctx2, layers, kv_len, target_token).
+    """
+
+    def __init__(self, step, example, bind):
+        self.step = step
+        dev = step.device
+        self.shapes = [(t.shape, t.dtype) for t in example]
+        self.offs, pos = [], 0
+        for t in example:
+            self.offs.append(pos)
+            pos += -(-t.numel() * t.element_size() // 256) * 256
+        self.nbytes = pos
+        self.staging = [torch.empty(pos, dtype=torch.uint8, device=dev) for _ in range(2)]
+        self.graphs = [step.capture(*bind(self.views(s))) for s in self.staging]
+        self.copy_stream = torch.cuda.Stream(device=dev)
+        self.result_host = [torch.empty(step.result.numel(), dtype=step.result.dtype).pin_memory()
+                            for _ in range(2)]
+        self.copied = [torch.cuda.Event(), torch.cuda.Event()]  # inputs in staging[s]
+        self.done = [torch.cuda.Event(), torch.cuda.Event()]    # round on staging[s] finished
+        self.read = [torch.cuda.Event(), torch.cuda.Event()]    # results in result_host[s]
+        self.pending = None
+
+    def views(self, buf):
+        return [buf[o:o + torch.Size(sh).numel() * torch.empty(0, dtype=dt).element_size()]
+                .view(dt).view(sh) for o, (sh, dt) in zip(self.offs, self.shapes)]
+
+    def pack(self, tensors):
+        """One round's inputs, packed into a new pinned host buffer."""
+        hb = torch.empty(self.nbytes, dtype=torch.uint8).pin_memory()
+        for v, t in zip(self.views(hb), tensors):
+            v.copy_(t.cpu())
+        return hb
+
+    def _upload(self, host_buf, s):
+        cs = self.copy_stream
+        cs.wait_event(self.done[s])  # the round that last read staging[s] has finished
+        with torch.cuda.stream(cs):
+            self.staging[s].copy_(host_buf, non_blocking=True)
+        self.copied[s].record(cs)
+
+    def start(self, host_buf):
+        """Queue the first round's inputs (into staging buffer 0)."""
+        self._upload(host_buf, 0)
+
+    def run(self, i, next_host_buf=None):
+        """Run round i (its inputs queued by start() or the previous run()), queue
+        next_host_buf for round i + 1, and return round i's results on the host."""
+        s = i % 2
+        main = torch.cuda.current_stream(self.step.device)
+        main.wait_event(self.copied[s])
+        self.graphs[s].replay()
+        self.done[s].record(main)
+        self.result_host[s].copy_(self.step.result, non_blocking=True)
+        self.read[s].record(main)
+        if next_host_buf is not None:
+            self._upload(next_host_buf, s ^ 1)
+        self.read[s].synchronize()
+        return self.result_host[s]

@@ -103,6 +103,10 @@ def test_host_validation_rejects_bad_arguments():
     # table: capacity out of range
     bad = _lib.Ngram3(16, 16, 40, -12.0)
     assert lib.presto_ngram3_clear(ctypes.byref(bad), N) == -1
+    # wait self-test: a status word is required; the limit stays within the library's
+    assert lib.presto_selftest_wait_timeout(N, 1000, N) == -1
+    assert lib.presto_selftest_wait_timeout(p, -1, N) == -1
+    assert lib.presto_selftest_wait_timeout(p, 3_000_000_000, N) == -1
 
 
 def test_binding_raises_on_error_status():

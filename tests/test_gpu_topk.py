@@ -112,3 +112,16 @@ def test_topk_stream_ties_masks_and_adversarial_rows():
     y[1, :5] = torch.linspace(-20, 20, 70000)                   # increasing rows
     y[2, :5] = torch.linspace(20, -20, 70000)                   # decreasing rows
     assert _check(y, 12) == 0
+
+
+@pytest.mark.parametrize("dtype,Vw,off,V,k", [(torch.float32, 70008, 3, 70003, 11),
+                                              (torch.bfloat16, 151944, 5, 151937, 8)])
+def test_topk_streaming_plan_misaligned_base_and_tail(dtype, Vw, off, V, k):
+    """Many long rows (the streaming plan: equal pieces that cross row boundaries,
+    partials merged per row) whose base is not 16-byte aligned while the row stride
+    is: every row has the same few head elements before its first aligned vector and
+    a tail after its last."""
+    g = torch.Generator().manual_seed(Vw + off)
+    wide = (torch.randn(4, 32, Vw, generator=g) * 3).to(dtype)
+    sub = wide[:, :, off:off + V].contiguous()
+    assert _check(sub, k, view=lambda t, w=wide: w.cuda()[:, :, off:off + V]) == 0

@@ -289,10 +289,10 @@ def oracle_check(w, gpu_file):
                                 "shapes": [list(mask.shape), list(g["mask"].shape)]}
     c["pos_ids"] = bool(np.array_equal(pos, g["pos_ids"]))
     if w.layers == 1:
-        att = synth.attention_inputs(w, device="cpu")
-        f64 = lambda x: x.double().numpy()
-        out, _ = O.tree_attention(f64(att["q"]), f64(att["k_cache"]), f64(att["v_cache"]),
-                                  g["kv_len"], f64(att["k_tree"]), f64(att["v_tree"]),
+        # the layer's Q / K / V exactly as the GPU read them (bf16 widened to float32)
+        f64 = lambda x: np.asarray(x, np.float64)
+        out, _ = O.tree_attention(f64(g["q"]), f64(g["k_cache"]), f64(g["v_cache"]),
+                                  g["kv_len"], f64(g["k_tree"]), f64(g["v_tree"]),
                                   g["mask"], g["n_nodes"])
         c["attention_max_abs"] = float(np.abs(out - g["attn"]).max())
     else:
@@ -629,6 +629,9 @@ def round_parity(w, step, st0, graph0, oracle_file):
          "accept_path": h(step.accept_path), "bonus": h(step.bonus), "target": h(st0["target"]),
          "kv_len": h(st0["kv_len"])}
     g.update({k: h(v) for k, v in step.tree.items()})
+    if w.layers == 1:  # the attention inputs are drawn on the GPU: hand them over as read
+        g.update({k: h(st0["layers"][0][k].float()) for k in ("q", "k_cache", "v_cache",
+                                                               "k_tree", "v_tree")})
     c = {"topk_ids": bool(np.array_equal(g["ids"], o["ids"])),
          "logq_rel_err": rel(g["logq"], o["logq"]),
          "lse_rel_err": rel(h(step.lse).reshape(R), o["lse"]),

@@ -19,7 +19,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OBJDIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libpresto.so")
-SOURCES = ["api.cu", "topk.cu", "tree_build.cu", "tree_mask_accept.cu", "tree_attention.cu"]
+SOURCES = ["api.cu", "topk.cu", "tree_build.cu", "tree_mask_accept.cu", "tree_attention.cu",
+           "tree_attention_pair.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
                 "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]

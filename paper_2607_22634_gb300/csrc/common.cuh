@@ -303,6 +303,15 @@ inline cudaLaunchAttribute pdl_attribute() {
   return at;
 }
 
+// Loads of data that an earlier kernel of the stream writes (read after the grid
+// dependency wait) go through L2 only.  Kernels of a dependent-launch chain start
+// while earlier ones still run, so an SM's L1 can hold lines that a previous
+// instance of a kernel read before they were rewritten; L2 is coherent.
+template <typename T>
+__device__ __forceinline__ T ld_chain(const T* p) {
+  return __ldcg(p);
+}
+
 __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));

@@ -221,9 +221,9 @@ __device__ __forceinline__ const T* row_base(const Args& a, int row, bool first)
   const T* base = static_cast<const T*>(a.logits);
   if (!a.acc_len) return base + static_cast<long long>(row) * a.row_stride;
   const int b = row / a.Lrows, j = row - b * a.Lrows;
-  const int len = a.acc_len[b];
+  const int len = ld_chain(a.acc_len + b);
   int node = -1;
-  if (len >= 0 && len < a.path_len) node = a.acc_path[static_cast<long long>(b) * a.path_len + len];
+  if (len >= 0 && len < a.path_len) node = ld_chain(a.acc_path + static_cast<long long>(b) * a.path_len + len);
   if (node < 0 || node >= a.n_prev) {
     if (first) report(a.dev_status, PRESTO_DEV_BAD_PATH);
     node = 0;

@@ -4,27 +4,28 @@
 //
 // The GQA group of one kv head (G = Hq/Hkv query heads x N nodes = G*N rows) is a
 // dense contraction against that head's keys, so it runs on the 5th-generation
-// tensor cores, ping-ponging two 128-row tiles per CTA:
-//   * one CTA per (sequence, kv head, pair of 128-row tiles, KV split);
-//   * warp 8 loads both Q tiles, then K tiles of 128 keys into a ring; warp 10 loads
-//     V tiles into another (TMA, 128-byte swizzle; 2 stages each at D = 128).  A K
-//     slot is refilled once both QK^T products of its tile completed, a V slot once
-//     both PV products did;
-//   * warp 9 issues tcgen05.mma: S_t = Q_t K^T (128 fp32 TMEM columns per row tile)
-//     and O_t += P_t V with P_t (bf16) read from TMEM, where the softmax wrote it over
-//     S_t.  Per KV tile: PV(t0), QK^T(t0) of the next tile, PV(t1), QK^T(t1); each
-//     QK^T waits for the completion of the PV that read the same TMEM, and the two
-//     row tiles ping-pong so that one tile's softmax overlaps the other tile's
-//     tensor work.  The whole warp runs the issue loop and one elected lane issues,
-//     so descriptors stay on the uniform datapath;
-//   * warps 0-3 and 4-7 run the softmax of tiles 0 and 1, one thread per query row
-//     (TMEM lane): the row's 128 scores in registers (four tcgen05.ld in flight),
-//     prefix-length and ancestor-bitmask masks (full prefix tiles skip them), online
-//     softmax with packed fp32x2 arithmetic, P written back over S with tcgen05.st.
-//     The running maximum is only moved (and O rescaled in TMEM) when it grows by
-//     more than 2^8, so most tiles skip the rescale;
-//   * with several KV splits (a row block's prefix and tree-key tiles dealt out in
-//     equal runs), the splits of one row block form a thread-block cluster (up to 16
+// tensor cores:
+//   * one CTA per (sequence, kv head, 128-row tile, KV split);
+//   * warp 8 loads the Q tile, then K tiles of 128 keys into a ring; warp 10 loads V
+//     tiles into another (TMA, 128-byte swizzle);
+//   * warp 9 issues tcgen05.mma: S_j = Q K_j^T into one of three 128-column TMEM
+//     buffers (j mod 3), and O += P_j V_j with P_j (bf16) read from TMEM, where the
+//     softmax wrote it over S_j.  QK^T runs up to three KV tiles ahead of PV: the
+//     QK^T of tile j + 3 is issued once the PV of tile j (the last reader of that
+//     buffer) has completed, so the softmax of the next tiles never waits for the
+//     tensor core's commit latency.  The whole warp runs the issue loop and one
+//     elected lane issues, so descriptors stay on the uniform datapath;
+//   * warps 0-7 run the softmax, two threads per query row (TMEM lane): warps 0-3
+//     take score columns 0-63, warps 4-7 columns 64-127 of the same rows.  Each
+//     thread masks its 64 scores (prefix length; ancestor bitmask for tree keys; full
+//     prefix tiles skip both), the pair combines its row maximum through shared
+//     memory (a barrier that also makes a timed-out wait a decision of all eight
+//     warps), then exponentiates with packed fp32x2 arithmetic and writes its half
+//     of P back over S with tcgen05.st.  The running maximum only moves (and O is
+//     rescaled in TMEM, after the previous PV completed) when it grows by more than
+//     2^8, so most tiles skip the rescale;
+//   * with several KV splits (a row tile's prefix and tree-key tiles dealt out in
+//     equal runs), the splits of one row tile form a thread-block cluster (up to 16
 //     CTAs): each CTA writes its rows' fp32 (m, l) and O / l to the workspace (bf16
 //     column quads, or float32 column pairs when the prefix is short; coalesced
 //     either way), the cluster synchronises (release / acquire), and each CTA
@@ -49,23 +50,25 @@ namespace {
 
 constexpr int kBM = 128;        // query rows per tile (TMEM lanes)
 constexpr int kBN = 128;        // keys per KV tile
-// 11 warps: 0-3 and 4-7 run the softmax of row tiles 0 and 1 (one thread per query
-// row = TMEM lane), 8 loads Q and K, 9 issues tensor-core MMAs, 10 loads V
+// 11 warps: 0-7 run the softmax (two threads per query row: warps q and q + 4 share
+// TMEM lane quadrant q), 8 loads Q and K, 9 issues tensor-core MMAs, 10 loads V
 constexpr int kThreads = 352;
 constexpr int kKWarp = 8;
 constexpr int kMmaWarp = 9;
 constexpr int kVWarp = 10;
-constexpr int kSoftThreads = 128;  // per tile
+constexpr int kSoftWarps = 8;
+constexpr int kSoftBar = 1;      // named barrier of the softmax warps
+constexpr int kSBufs = 3;        // S buffers in TMEM
 constexpr float kRescaleLog2 = 8.f;  // move the running max only when it grows by > 2^8
 constexpr int kRowBytes = 128;       // one 128-byte-swizzled row: 64 bf16
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
-// TMEM columns: S of tile t (128 fp32) at 128t, overwritten in place by P of tile t
-// (128 bf16 packed in pairs, its first 64 columns); O of tile t at 256 + 128t
+// TMEM columns: S buffer s (128 fp32) at 128 s, overwritten in place by P (128 bf16
+// packed in pairs, its first 64 columns); O (D fp32) at 384
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kTmemO = 256;
+constexpr uint32_t kTmemO = 128 * kSBufs;
 constexpr int kWidePartialKeys = 1024;  // prefixes shorter than this merge float32 partials
-constexpr int kMaxSplits = 16;  // KV splits of a row block = CTAs of its cluster
+constexpr int kMaxSplits = 16;  // KV splits of a row tile = CTAs of its cluster
 
 struct Args {
   const __nv_bfloat16* k_cache;  // [B, Hkv, Tmax, D] (for the L2 prefetch)
@@ -73,29 +76,29 @@ struct Args {
   const int32_t* kv_len;
   const uint32_t* mask;
   const int32_t* n_nodes;
-  int B, N, Hq, Hkv, G, Tmax, W, n_mt, tpc, n_groups, n_splits;  // tpc: row tiles per CTA
+  int B, N, Hq, Hkv, G, Tmax, W, n_mt, n_splits;
   float scale_log2;
   __nv_bfloat16* out;
   float* lse;
-  float2* part_o;   // KV splits: O / l of each row, float32 [CTA][D / 2][2 * kBM] (column pairs)
-  float2* part_ml;  // KV splits: (m, l) per row [CTA][2 * kBM], log2 domain
+  float2* part_o;   // KV splits: O / l of each row, [CTA][column group][kBM]
+  float2* part_ml;  // KV splits: (m, l) per row [CTA][kBM], log2 domain
   int32_t* dev_status;
 };
 
-// Shared memory: Q of both row tiles, the K ring, the V ring.  Every operand is
-// stored as 64-column panels of 128-byte rows with the 128-byte swizzle (128 rows
-// per panel).  Ring depths: 2 at D = 128 (192 KB in all), 4 at D = 64.
+// Shared memory: the Q tile, the K ring, the V ring.  Every operand is stored as
+// 64-column panels of 128-byte rows with the 128-byte swizzle (128 rows per panel).
+// Ring depths: K 2 and V 3 at D = 128 (192 KB in all), 4 and 4 at D = 64.
 template <int D>
 struct Layout {
   static constexpr int kKStages = D == 64 ? 4 : 2;
-  static constexpr int kVStages = D == 64 ? 4 : 2;
+  static constexpr int kVStages = D == 64 ? 4 : 3;
   static constexpr int kPanels = D / 64;
   static constexpr int kQPanel = kBM * kRowBytes;   // 16 KB
   static constexpr int kKVPanel = kBN * kRowBytes;  // 16 KB
   static constexpr int kQBytes = kBM * D * 2;
   static constexpr int kTileBytes = kBN * D * 2;    // one K or V tile
-  static constexpr int kQ = 0;                          // tile 0, then tile 1
-  static constexpr int kK = kQ + 2 * kQBytes;
+  static constexpr int kQ = 0;
+  static constexpr int kK = kQ + kQBytes;
   static constexpr int kV = kK + kKStages * kTileBytes;
   static constexpr int kBytes = kV + kVStages * kTileBytes;
   static constexpr int kAlloc = kBytes + 1024;  // room to align the base to 1024
@@ -106,9 +109,26 @@ struct Bars {
   uint64_t q_full;
   uint64_t k_full[kMaxStages], k_empty[kMaxStages];
   uint64_t v_full[kMaxStages], v_empty[kMaxStages];
-  uint64_t s_full[2], p_full[2], o_done[2];
-  uint64_t drain;  // after a timed-out wait: every MMA issued so far has completed
+  uint64_t s_full[kSBufs], p_full[kSBufs];
+  uint64_t o_done;  // one phase per PV: O holds the products of tiles 0..j
+  uint64_t drain;   // after a timed-out wait: every MMA issued so far has completed
 };
+
+// The softmax warps' barrier with an AND over their predicates: every one of the
+// 256 threads arrives, and all leave with the same answer.
+__device__ __forceinline__ bool soft_sync_and(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.u32 q, %1, 0;\n bar.red.and.pred p, %2, %3, q;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(v)), "n"(kSoftBar), "n"(kSoftWarps * 32)
+      : "memory");
+  return r != 0;
+}
+__device__ __forceinline__ void soft_sync() {
+  asm volatile("bar.sync %0, %1;" ::"n"(kSoftBar), "n"(kSoftWarps * 32) : "memory");
+}
 
 // Packed fp32 pairs (f32x2 arithmetic issues one instruction per two values) and
 // the three-input max.
@@ -160,6 +180,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ Bars bars;
   __shared__ uint32_t tmem_base;
   __shared__ int abort_flag;
+  __shared__ float xmax[2][2][kBM];  // per iteration parity and half: the half-row maxima
+  __shared__ float xl[2][kBM];       // per half: the half-row sums
   __shared__ float mw[kBM][kMaxSplits + 1];  // split merge: per-row weights (slice <= kBM rows)
   __shared__ float mlse[kBM];                // split merge: per-row lse
 
@@ -167,13 +189,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   int idx = blockIdx.x;
   const int split = idx % a.n_splits;
   idx /= a.n_splits;
-  const int mp = idx % a.n_groups;  // group of a.tpc row tiles
-  idx /= a.n_groups;
+  const int mt = idx % a.n_mt;  // row tile
+  idx /= a.n_mt;
   const int g = idx % a.Hkv;
   const int b = idx / a.Hkv;
-  const int mt0 = mp * a.tpc;       // first row tile of the group
-  const bool has1 = a.tpc == 2 && mt0 + 1 < a.n_mt;  // second tile present
-  const int ntiles = has1 ? 2 : 1;
   const bool clustered = a.n_splits > 1;
   const int nodes_per_tile = kBM / a.G;
   pdl_launch_dependents();
@@ -186,11 +205,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bars.v_full[st], 1);
       mbar_init(&bars.v_empty[st], 1);
     }
-    for (int t = 0; t < 2; ++t) {
-      mbar_init(&bars.s_full[t], 1);
-      mbar_init(&bars.p_full[t], kSoftThreads);
-      mbar_init(&bars.o_done[t], 1);
+    for (int s = 0; s < kSBufs; ++s) {
+      mbar_init(&bars.s_full[s], 1);
+      mbar_init(&bars.p_full[s], kSoftWarps);
     }
+    mbar_init(&bars.o_done, 1);
     mbar_init(&bars.drain, 1);
     abort_flag = 0;
     fence_barrier_init();
@@ -224,8 +243,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   pdl_wait();  // the mask and node counts come from the previous kernels on the stream
-  const int kv_raw = a.kv_len[b];
-  const int nn_raw = a.n_nodes[b];
+  const int kv_raw = ld_chain(a.kv_len + b);
+  const int nn_raw = ld_chain(a.n_nodes + b);
 
   int kv = kv_raw;
   if (kv < 0 || kv > a.Tmax) {
@@ -239,7 +258,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   // a long prefix bf16 partials (half the merge traffic) lose nothing measurable
   const bool wide = kv < kWidePartialKeys;
   const int prefix_tiles = (kv + kBN - 1) / kBN;
-  // the KV tiles of a row block, prefix tiles then tree tiles, in equal runs over the
+  // the KV tiles of a row tile, prefix tiles then tree tiles, in equal runs over the
   // splits: this split's local tile j is prefix tile t_begin + j for j < n_prefix,
   // else tree tile tree0 + (j - n_prefix)
   const int tree_tiles = (nn + kBN - 1) / kBN;
@@ -263,12 +282,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tensormap(&tm_q);
       prefetch_tensormap(&tm_kc);
       prefetch_tensormap(&tm_kt);
-      mbar_arrive_expect_tx(&bars.q_full, ntiles * Ly::kQBytes);
-      for (int t = 0; t < ntiles; ++t)
-        for (int p = 0; p < Ly::kPanels; ++p)
-          tma_load_3d(smem + Ly::kQ + t * Ly::kQBytes + p * Ly::kQPanel, &tm_q, p * 64, g * a.G,
-                      b * a.N + (mt0 + t) * nodes_per_tile, &bars.q_full);
-      // K_j -> slot j % Ly::kKStages, once both QK^T of K_{j - Ly::kKStages} completed
+      mbar_arrive_expect_tx(&bars.q_full, Ly::kQBytes);
+      for (int p = 0; p < Ly::kPanels; ++p)
+        tma_load_3d(smem + Ly::kQ + p * Ly::kQPanel, &tm_q, p * 64, g * a.G, b * a.N + mt * nodes_per_tile,
+                    &bars.q_full);
+      // K_j -> slot j % Ly::kKStages, once the QK^T of K_{j - Ly::kKStages} completed
       for (int j = 0; j < nt; ++j) {
         const int st = j % Ly::kKStages;
         if (j >= Ly::kKStages && !mbar_wait(&bars.k_empty[st], (j / Ly::kKStages - 1) & 1, abort)) {
@@ -293,7 +311,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       prefetch_tensormap(&tm_vc);
       prefetch_tensormap(&tm_vt);
-      // V_j -> slot j % Ly::kVStages, once both PV of V_{j - Ly::kVStages} completed
+      // V_j -> slot j % Ly::kVStages, once the PV of V_{j - Ly::kVStages} completed
       for (int j = 0; j < nt; ++j) {
         const int st = j % Ly::kVStages;
         if (j >= Ly::kVStages && !mbar_wait(&bars.v_empty[st], (j / Ly::kVStages - 1) & 1, abort)) {
@@ -315,13 +333,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (nt > 0 && warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
-    // Per KV tile j and row tile t: PV_j(t) (P_t read from TMEM, where it overwrote
-    // S_t), then QK_{j+1}(t) into the same TMEM, issued once PV_j(t) has completed
-    // (its o_done), so S_t is never rewritten while P_t is still being read.  The whole warp runs this loop (wait outcomes made
-    // warp-uniform); one elected lane issues each MMA and commit.
+    // S_j goes to TMEM buffer j % 3.  The first three QK^T are issued as their K tiles
+    // land; then per tile j: PV_j once P_j is written (P_j read from buffer j % 3),
+    // and QK^T of tile j + 3 into the same buffer once PV_j has completed (o_done),
+    // so S is never rewritten while P is still being read.  The whole warp runs this
+    // loop (wait outcomes made warp-uniform); one elected lane issues each MMA and
+    // commit.
     constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, false);
     constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, true);
-    const uint64_t q_desc0 = smem_desc_sw128(smem_u32(smem + Ly::kQ), 16, 1024);
+    const uint64_t q_desc = smem_desc_sw128(smem_u32(smem + Ly::kQ), 16, 1024);
     const uint64_t k_desc0 = smem_desc_sw128(smem_u32(smem + Ly::kK), 16, 1024);
     const uint64_t v_desc0 = smem_desc_sw128(smem_u32(smem + Ly::kV), Ly::kKVPanel, 1024);
     auto wait = [&](uint64_t* bar, uint32_t parity) {
@@ -329,122 +349,123 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (ok) tc_fence_after();
       return ok;
     };
-    // S_t = Q_t K_j^T
-    auto qk = [&](int t, int j) {
+    // S_j = Q K_j^T (K_j resident)
+    auto qk = [&](int j) {
+      const int s = j % kSBufs;
       // descriptor start addresses are in 16-byte units in the low bits
-      const uint64_t qd = q_desc0 + ((t * Ly::kQBytes) >> 4);
       const uint64_t kd = k_desc0 + (((j % Ly::kKStages) * Ly::kTileBytes) >> 4);
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t qo = ((kk >> 2) * Ly::kQPanel + (kk & 3) * 32) >> 4;
         const uint32_t ko = ((kk >> 2) * Ly::kKVPanel + (kk & 3) * 32) >> 4;
-        mma_bf16_warp(tmem_base + t * 128, qd + qo, kd + ko, idesc_qk, kk > 0);
+        mma_bf16_warp(tmem_base + s * 128, q_desc + qo, kd + ko, idesc_qk, kk > 0);
       }
-      mma_commit_warp(&bars.s_full[t]);
+      mma_commit_warp(&bars.s_full[s]);
+      mma_commit_warp(&bars.k_empty[j % Ly::kKStages]);
     };
-    // O_t (+)= P_t V_j, P_t read from TMEM (8 columns = 16 keys per step)
-    auto pv = [&](int t, int j) {
-      if (!wait(&bars.p_full[t], j & 1)) return false;
+    // O (+)= P_j V_j, P_j read from TMEM (8 columns = 16 keys per step)
+    auto pv = [&](int j) {
+      const int s = j % kSBufs;
+      if (!wait(&bars.p_full[s], (j / kSBufs) & 1)) return false;
       const uint64_t vd = v_desc0 + (((j % Ly::kVStages) * Ly::kTileBytes) >> 4);
 #pragma unroll
       for (int kk = 0; kk < kBN / 16; ++kk)
-        mma_bf16_ts_warp(tmem_base + kTmemO + t * 128, tmem_base + t * 128 + kk * 8,
+        mma_bf16_ts_warp(tmem_base + kTmemO, tmem_base + s * 128 + kk * 8,
                          vd + ((kk * 16 * kRowBytes) >> 4), idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
-      mma_commit_warp(&bars.o_done[t]);
+      mma_commit_warp(&bars.o_done);
+      mma_commit_warp(&bars.v_empty[j % Ly::kVStages]);
       return true;
     };
-    bool ok = wait(&bars.q_full, 0) && wait(&bars.k_full[0], 0);
-    if (ok) {
-      qk(0, 0);
-      if (has1) qk(1, 0);
-      mma_commit_warp(&bars.k_empty[0]);
+    bool ok = wait(&bars.q_full, 0);
+    for (int j = 0; ok && j < min(nt, kSBufs); ++j) {
+      ok = wait(&bars.k_full[j % Ly::kKStages], (j / Ly::kKStages) & 1);
+      if (ok) qk(j);
     }
-    // ping-pong: tile 0's next S is issued right after its PV, so its softmax runs
-    // while the tensor core works on tile 1, and the other way round
     for (int j = 0; ok && j < nt; ++j) {
-      const int jn = j + 1;
-      const bool more = jn < nt;
-      ok = wait(&bars.v_full[j % Ly::kVStages], (j / Ly::kVStages) & 1) && pv(0, j);
-      if (ok && more) {
-        ok = wait(&bars.k_full[jn % Ly::kKStages], (jn / Ly::kKStages) & 1) &&
-             wait(&bars.o_done[0], j & 1);
-        if (ok) qk(0, jn);
+      ok = wait(&bars.v_full[j % Ly::kVStages], (j / Ly::kVStages) & 1) && pv(j);
+      const int jn = j + kSBufs;
+      if (ok && jn < nt) {
+        ok = wait(&bars.o_done, j & 1) &&
+             wait(&bars.k_full[jn % Ly::kKStages], (jn / Ly::kKStages) & 1);
+        if (ok) qk(jn);
       }
-      if (ok && has1) {
-        ok = pv(1, j);
-        if (ok && more) {
-          ok = wait(&bars.o_done[1], j & 1);
-          if (ok) qk(1, jn);
-        }
-      }
-      if (!ok) break;
-      mma_commit_warp(&bars.v_empty[j % Ly::kVStages]);
-      if (more) mma_commit_warp(&bars.k_empty[jn % Ly::kKStages]);
     }
     if (!ok && lane == 0) fail();
-  } else if (nt > 0 && warp < 4 * ntiles) {
+  } else if (nt > 0 && warp < kSoftWarps) {
     // ------------------------------------------------------------ softmax warps
-    const int t = warp >> 2;          // row tile
     const int quad = warp & 3;        // TMEM lane quadrant
+    const int h = warp >> 2;          // half of the score columns: 64 h .. 64 h + 63
     const int r = quad * 32 + lane;   // row of the tile
     const uint32_t lane_addr = static_cast<uint32_t>(quad * 32) << 16;
-    const uint32_t tO = tmem_base + kTmemO + t * 128 + lane_addr;
-    const uint32_t tS = tmem_base + t * 128 + lane_addr;  // S_t, then P_t in place
-    const int node = (mt0 + t) * nodes_per_tile + r / a.G;
-    const int hh = r % a.G;
+    const uint32_t tO = tmem_base + kTmemO + lane_addr;
+    const int node = mt * nodes_per_tile + r / a.G;
     const uint32_t* mrow =
         node < a.N ? a.mask + (static_cast<size_t>(b) * a.N + node) * a.W : nullptr;
-    float m = -INFINITY, l = 0.f;  // m: running (possibly stale) max, log2 domain
+    float m = -INFINITY, l = 0.f;  // m: running (possibly stale) max, log2 domain; l: this half's sum
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
-      // wait outcomes are made warp-uniform: tcgen05.ld needs the whole warp.  S_j
-      // ready also means PV_{j-1} of this tile completed (QK_j was issued after it),
-      // so O_t may be rescaled and P_t rewritten.
-      if (!__all_sync(0xffffffffu, mbar_wait(&bars.s_full[t], j & 1, abort))) {
+      const int s = j % kSBufs;
+      const uint32_t tS = tmem_base + s * 128 + lane_addr;  // S_j, then P_j in place
+      // wait outcomes are warp-uniform (tcgen05.ld needs the whole warp) and then
+      // shared by all eight warps at the exchange barrier below
+      bool got = ok && __all_sync(0xffffffffu, mbar_wait(&bars.s_full[s], (j / kSBufs) & 1, abort));
+      if (ok && !got) fail();  // the other warps' waits end at once
+      float v[64];
+      float mx = -INFINITY;
+      const bool full = j < n_prefix && kv - (t_begin + j) * kBN >= kBN;  // CTA-uniform
+      if (got) {
+        tc_fence_after();
+        // masks of this half's two 32-key chunks: prefix keys beyond kv_len; tree keys
+        // outside the ancestor set (a full prefix tile needs none)
+        uint32_t bits[2];
+        if (j < n_prefix) {
+          const int lim = kv - (t_begin + j) * kBN - 64 * h;
+#pragma unroll
+          for (int c = 0; c < 2; ++c) {
+            const int lc = lim - 32 * c;
+            bits[c] = lc >= 32 ? 0xffffffffu : (lc <= 0 ? 0u : (1u << lc) - 1u);
+          }
+        } else {
+          const int wi = (((tree0 + j - n_prefix) * kBN) >> 5) + 2 * h;
+#pragma unroll
+          for (int c = 0; c < 2; ++c) bits[c] = (mrow && wi + c < a.W) ? ld_chain(mrow + wi + c) : 0u;
+        }
+        // this half's 64 scores: two loads in flight, one wait
+#pragma unroll
+        for (int c = 0; c < 2; ++c)
+          tmem_ld32(tS + 64 * h + c * 32, *reinterpret_cast<float(*)[32]>(v + 32 * c));
+        tmem_wait_ld();
+        if (!full) {  // masked scores -> -inf (exp2 of -inf is 0)
+#pragma unroll
+          for (int c = 0; c < 2; ++c)
+#pragma unroll
+            for (int e = 0; e < 32; ++e) v[32 * c + e] = ((bits[c] >> e) & 1u) ? v[32 * c + e] : -INFINITY;
+        }
+        mx = fmaxf(row_max32(v), row_max32(v + 32)) * a.scale_log2;  // scale > 0 commutes with max
+        xmax[j & 1][h][r] = mx;
+      }
+      // both halves' maxima are written and every load of S_j has completed (the
+      // other half overwrites part of this half's S columns with its P below)
+      tc_fence_before();
+      got = soft_sync_and(got);
+      tc_fence_after();
+      if (!got) {
         ok = false;
         break;
       }
-      tc_fence_after();
-      // masks of the four 32-key chunks: prefix keys beyond kv_len; tree keys outside
-      // the ancestor set (a full prefix tile needs none)
-      uint32_t bits[4];
-      const bool full = j < n_prefix && kv - (t_begin + j) * kBN >= kBN;  // warp-uniform
-      if (j < n_prefix) {
-        const int lim = kv - (t_begin + j) * kBN;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const int lc = lim - 32 * c;
-          bits[c] = lc >= 32 ? 0xffffffffu : (lc <= 0 ? 0u : (1u << lc) - 1u);
-        }
-      } else {
-        const int wi = ((tree0 + j - n_prefix) * kBN) >> 5;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) bits[c] = (mrow && wi + c < a.W) ? __ldg(mrow + wi + c) : 0u;
-      }
-      // the row's 128 scores: four loads in flight, one wait
-      float v[128];
-#pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(tS + c * 32, *reinterpret_cast<float(*)[32]>(v + 32 * c));
-      tmem_wait_ld();
-      if (!full) {  // masked scores -> -inf (exp2 of -inf is 0)
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
-#pragma unroll
-          for (int e = 0; e < 32; ++e) v[32 * c + e] = ((bits[c] >> e) & 1u) ? v[32 * c + e] : -INFINITY;
-      }
-      float mx = fmaxf(fmaxf(row_max32(v), row_max32(v + 32)), fmaxf(row_max32(v + 64), row_max32(v + 96)));
-      mx *= a.scale_log2;  // scale > 0 commutes with max
+      mx = fmaxf(mx, xmax[j & 1][h ^ 1][r]);
       // stale-max online softmax: move m only when the row max exceeds it by > 2^8
+      // (both halves of a row take the same decision)
       const bool move = mx > m + kRescaleLog2;
       const float alpha = move ? ex2(m - mx) : 1.f;
       if (move) m = mx;
       const float m_use = m == -INFINITY ? 0.f : m;
-      // p = exp2(s * scale - m), stored as bf16 pairs over the S columns (P covers the
-      // first 64, all of S having been read); the row sum in packed chains
+      // p = exp2(s * scale - m), stored as bf16 pairs over the S columns: this half's
+      // 64 keys are P columns 32 h .. 32 h + 31; the half-row sum in packed chains
       const uint64_t sc2 = pack2(a.scale_log2, a.scale_log2), nm2 = pack2(-m_use, -m_use);
       uint64_t acc[2] = {0ull, 0ull};
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
+      for (int c = 0; c < 2; ++c) {
         uint32_t pk[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
@@ -455,17 +476,26 @@ __global__ void __launch_bounds__(kThreads, 1)
           const __nv_bfloat162 pv2 = __floats2bfloat162_rn(p0, p1);
           pk[i] = *reinterpret_cast<const uint32_t*>(&pv2);
         }
-        tmem_st16(tS + c * 16, pk);
+        tmem_st16(tS + 32 * h + c * 16, pk);
       }
-      if (j > 0 && __any_sync(0xffffffffu, move)) {  // O_t *= alpha (rows that did not move: 1)
+      if (j > 0 && __any_sync(0xffffffffu, move)) {
+        // O *= alpha over this half's columns (rows that did not move: 1), once the
+        // PV of tile j - 1 has completed
+        if (__all_sync(0xffffffffu, mbar_wait(&bars.o_done, (j - 1) & 1, abort))) {
+          tc_fence_after();
 #pragma unroll 1
-        for (int c = 0; c < D / 32; ++c) {
-          float o[32];
-          tmem_ld32(tO + c * 32, o);
-          tmem_wait_ld();
+          for (int c = 0; c < D / 64; ++c) {
+            float o[32];
+            const uint32_t col = (D / 2) * h + c * 32;
+            tmem_ld32(tO + col, o);
+            tmem_wait_ld();
 #pragma unroll
-          for (int e = 0; e < 32; ++e) o[e] *= alpha;
-          tmem_st32(tO + c * 32, o);
+            for (int e = 0; e < 32; ++e) o[e] *= alpha;
+            tmem_st32(tO + col, o);
+          }
+        } else {
+          ok = false;  // the next exchange barrier makes it every warp's decision
+          fail();
         }
       }
       float rs, rs1;
@@ -473,62 +503,65 @@ __global__ void __launch_bounds__(kThreads, 1)
       l = l * alpha + (rs + rs1);
       tmem_wait_st();  // P (and a rescaled O) are in TMEM before the MMA is released
       tc_fence_before();
-      mbar_arrive(&bars.p_full[t]);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars.p_full[s]);
     }
-    if (ok)
-      ok = __all_sync(0xffffffffu, mbar_wait(&bars.o_done[t], (nt - 1) & 1, abort));
-    if (!ok) fail();
+    // the row's sum over both halves
+    xl[h][r] = l;
+    soft_sync();
+    l += xl[h ^ 1][r];
+    if (ok) {
+      ok = __all_sync(0xffffffffu, mbar_wait(&bars.o_done, (nt - 1) & 1, abort));
+      if (!ok) fail();
+    }
     if (clustered) {
-      // this split's unnormalised row and (m, l) for the merge (a failed or empty
-      // row is marked by m = -inf and contributes nothing)
-      const size_t prow = static_cast<size_t>(blockIdx.x) * 2 * kBM + t * kBM + r;
-      a.part_ml[prow] = ok ? make_float2(m, l) : make_float2(-INFINITY, 0.f);
+      // this split's normalised row and (m, l) for the merge (a failed or empty row
+      // is marked by m = -inf and contributes nothing); each half writes its columns
+      const size_t prow = static_cast<size_t>(blockIdx.x) * kBM + r;
+      if (h == 0) a.part_ml[prow] = ok ? make_float2(m, l) : make_float2(-INFINITY, 0.f);
       if (ok) {
         tc_fence_after();
         // the row normalised by its own l (values stay within the range of V), laid
         // out so that a warp's 32 rows of one column group are 256 contiguous bytes:
         // bf16 column quads, or float32 column pairs when the sequence's prefix is
-        // short (wide_partials)
+        // short (wide partials)
         const float inv = l > 0.f ? 1.f / l : 0.f;
-        if (wide) {
-          float2* dst = reinterpret_cast<float2*>(a.part_o) +
-                        static_cast<size_t>(blockIdx.x) * (D / 2) * 2 * kBM + t * kBM + r;
 #pragma unroll 1
-          for (int c = 0; c < D / 32; ++c) {
-            float o[32];
-            tmem_ld32(tO + c * 32, o);
-            tmem_wait_ld();
+        for (int cc = 0; cc < D / 64; ++cc) {
+          const int c = h * (D / 64) + cc;  // 32-column chunk of O
+          float o[32];
+          tmem_ld32(tO + c * 32, o);
+          tmem_wait_ld();
+          if (wide) {
+            float2* dst = reinterpret_cast<float2*>(a.part_o) +
+                          static_cast<size_t>(blockIdx.x) * (D / 2) * kBM + r;
 #pragma unroll
             for (int q = 0; q < 16; ++q)
-              dst[(c * 16 + q) * 2 * kBM] = make_float2(o[q * 2] * inv, o[q * 2 + 1] * inv);
-          }
-        } else {
-          uint2* dst = reinterpret_cast<uint2*>(a.part_o) +
-                       static_cast<size_t>(blockIdx.x) * (D / 4) * 2 * kBM + t * kBM + r;
-#pragma unroll 1
-          for (int c = 0; c < D / 32; ++c) {
-            float o[32];
-            tmem_ld32(tO + c * 32, o);
-            tmem_wait_ld();
+              dst[(c * 16 + q) * kBM] = make_float2(o[q * 2] * inv, o[q * 2 + 1] * inv);
+          } else {
+            uint2* dst = reinterpret_cast<uint2*>(a.part_o) +
+                         static_cast<size_t>(blockIdx.x) * (D / 4) * kBM + r;
 #pragma unroll
             for (int q = 0; q < 8; ++q) {
               const __nv_bfloat162 lo = __floats2bfloat162_rn(o[q * 4] * inv, o[q * 4 + 1] * inv);
               const __nv_bfloat162 hi = __floats2bfloat162_rn(o[q * 4 + 2] * inv, o[q * 4 + 3] * inv);
-              dst[(c * 8 + q) * 2 * kBM] = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
-                                                      *reinterpret_cast<const uint32_t*>(&hi));
+              dst[(c * 8 + q) * kBM] = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
+                                                  *reinterpret_cast<const uint32_t*>(&hi));
             }
           }
         }
       }
     } else if (ok) {
       tc_fence_after();
-      // the normalised bf16 row, 32 columns at a time, and its lse
+      // the normalised bf16 row (this half's columns), and its lse
+      const int hh = r % a.G;
       const bool used = node < a.N && node < nn && l > 0.f;
       const float inv = used ? 1.f / l : 0.f;
       __nv_bfloat16* orow =
           a.out + ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
 #pragma unroll 1
-      for (int c = 0; c < D / 32; ++c) {
+      for (int cc = 0; cc < D / 64; ++cc) {
+        const int c = h * (D / 64) + cc;
         float o[32];
         tmem_ld32(tO + c * 32, o);
         tmem_wait_ld();
@@ -547,7 +580,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      if (node < a.N && a.lse)
+      if (h == 0 && node < a.N && a.lse)
         a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] =
             used ? (m + log2f(l)) * kLn2 : -INFINITY;
     }
@@ -573,9 +606,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   if (!clustered) {
-    if (nt == 0 && tid < ntiles * kBM) {  // no keys at all: a zero row, lse -inf
-      const int t = tid / kBM, r = tid % kBM;
-      const int node = (mt0 + t) * nodes_per_tile + r / a.G, hh = r % a.G;
+    if (nt == 0 && tid < kBM) {  // no keys at all: a zero row, lse -inf
+      const int r = tid;
+      const int node = mt * nodes_per_tile + r / a.G, hh = r % a.G;
       if (node < a.N) {
         __nv_bfloat16* orow =
             a.out + ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
@@ -593,12 +626,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // ---------------------------------------------------------------- split merge
-  // The KV splits of this row block are the CTAs of the cluster; each has left its
-  // rows' (m, l) and unnormalised O in the workspace.  Rows are dealt out in slices,
+  // The KV splits of this row tile are the CTAs of the cluster; each has left its
+  // rows' (m, l) and normalised O in the workspace.  Rows are dealt out in slices,
   // one per CTA, and each CTA combines its slice over the splits with log-sum-exp
   // weights (the partials stay in L2).
-  if (nt == 0 && tid < ntiles * kBM)  // an empty split contributes nothing
-    a.part_ml[static_cast<size_t>(blockIdx.x) * 2 * kBM + tid] = make_float2(-INFINITY, 0.f);
+  if (nt == 0 && tid < kBM)  // an empty split contributes nothing
+    a.part_ml[static_cast<size_t>(blockIdx.x) * kBM + tid] = make_float2(-INFINITY, 0.f);
   tc_fence_before();
   __syncthreads();
   if (warp == kMmaWarp) {
@@ -607,14 +640,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   // release / acquire at cluster scope: every split's partial rows are visible
   cg::this_cluster().sync();
-  const int R = ntiles * kBM;
+  const int R = kBM;
   const int nsp = a.n_splits;
   const int slice = (R + nsp - 1) / nsp;
   const size_t cta0 = static_cast<size_t>(blockIdx.x - split);  // first CTA of the cluster
   const int r0 = split * slice;
   const int nr = max(0, min(R, r0 + slice) - r0);
   // One item = one row of the slice x one column group (a bf16 quad or a float32
-  // pair), rows fastest (coalesced partial loads).  Each thread's first two items are
+  // pair), rows fastest (coalesced partial loads).  Each thread's first item is
   // loaded before the per-row weights are formed (one thread per row, into shared
   // memory), so the usual case costs one L2 round trip.
   auto merge = [&](auto wide_tag) {
@@ -624,15 +657,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     const PT* part = reinterpret_cast<const PT*>(a.part_o);
     const int nitems = nr * kCG;
     auto load_item = [&](int item, PT (&o)[kMaxSplits]) {
-      const int cg = item / nr, row = r0 + item % nr;
+      const int cg = item / max(nr, 1), row = r0 + item % max(nr, 1);
 #pragma unroll
       for (int s = 0; s < kMaxSplits; ++s)
-        o[s] = (item < nitems && s < nsp) ? __ldcg(part + ((cta0 + s) * kCG + cg) * 2 * kBM + row)
+        o[s] = (item < nitems && s < nsp) ? __ldcg(part + ((cta0 + s) * kCG + cg) * kBM + row)
                                          : PT{};
     };
-    PT oa[kMaxSplits], ob[kMaxSplits];
+    PT oa[kMaxSplits];
     load_item(tid, oa);
-    load_item(tid + kThreads, ob);
     if (tid < nr) {
       // the row's weights over the splits, w_s l_s / L (a split without keys for the
       // row has m = -inf and weight 0), and its lse
@@ -640,21 +672,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       float2 ml[kMaxSplits];
 #pragma unroll
       for (int s = 0; s < kMaxSplits; ++s)
-        ml[s] = s < nsp ? __ldcg(a.part_ml + (cta0 + s) * 2 * kBM + row) : make_float2(-INFINITY, 0.f);
+        ml[s] = s < nsp ? __ldcg(a.part_ml + (cta0 + s) * kBM + row) : make_float2(-INFINITY, 0.f);
       float M = -INFINITY;
 #pragma unroll
       for (int s = 0; s < kMaxSplits; ++s) M = fmaxf(M, ml[s].x);
-      float wl[kMaxSplits], L = 0.f;
+      float L = 0.f;
 #pragma unroll
       for (int s = 0; s < kMaxSplits; ++s) {
-        wl[s] = (M == -INFINITY || ml[s].x == -INFINITY) ? 0.f : ex2(ml[s].x - M) * ml[s].y;
-        L += wl[s];
+        const float wl = (M == -INFINITY || ml[s].x == -INFINITY) ? 0.f : ex2(ml[s].x - M) * ml[s].y;
+        mw[tid][s] = wl;
+        L += wl;
       }
-      const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
+      const int node = mt * nodes_per_tile + row / a.G;
       const bool used = node < nn && L > 0.f;
       const float inv = used ? 1.f / L : 0.f;
 #pragma unroll
-      for (int s = 0; s < kMaxSplits; ++s) mw[tid][s] = wl[s] * inv;
+      for (int s = 0; s < kMaxSplits; ++s) mw[tid][s] *= inv;
       mlse[tid] = used ? (M + log2f(L)) * kLn2 : -INFINITY;
     }
     __syncthreads();
@@ -662,8 +695,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (item >= nitems) return;
       const int cg = item / nr, i = item % nr;
       const int row = r0 + i;
-      const int node = (mt0 + row / kBM) * nodes_per_tile + (row % kBM) / a.G;
-      const int hh = (row % kBM) % a.G;
+      const int node = mt * nodes_per_tile + row / a.G;
+      const int hh = row % a.G;
       if (node >= a.N) return;
       float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
@@ -695,8 +728,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (cg == 0 && a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = mlse[i];
     };
     finish_item(tid, oa);
-    finish_item(tid + kThreads, ob);
-    for (int item = tid + 2 * kThreads; item < nitems; item += kThreads) {
+    for (int item = tid + kThreads; item < nitems; item += kThreads) {
       load_item(item, oa);
       finish_item(item, oa);
     }
@@ -737,10 +769,9 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64
 }
 
 struct Plan {
-  int G, n_mt, tpc, n_groups, n_splits;
+  int G, n_mt, n_splits;
   size_t ctas;
 };
-
 
 // active[s] = how many clusters of s CTAs (s = 1..kMaxSplits) can be resident on
 // the GPU at once; 0 where that cluster size does not fit.
@@ -748,36 +779,27 @@ Plan make_plan(int B, int N, int Hq, int Hkv, int Tmax, const int* active) {
   Plan p;
   p.G = Hq / Hkv;
   p.n_mt = (N * p.G + kBM - 1) / kBM;
-  const int prefix_tiles = (Tmax + kBN - 1) / kBN;
-  const int tree_tiles = (N + kBN - 1) / kBN;
-  int max_splits = (prefix_tiles + tree_tiles) / 2 > 1 ? (prefix_tiles + tree_tiles) / 2 : 1;
+  const int tiles = (Tmax + kBN - 1) / kBN + (N + kBN - 1) / kBN;
+  int max_splits = tiles / 2 > 1 ? tiles / 2 : 1;
   if (max_splits > kMaxSplits) max_splits = kMaxSplits;
-  // Choose row tiles per CTA (2 lets the softmax of one tile hide behind the
-  // tensor-core work of the other, and reads K/V once for both) and the split
-  // count by the estimated time: waves of resident clusters x (KV tiles per CTA x
-  // cost of one KV tile + fixed cost), lightly penalising splits (each adds rows
-  // to merge).
+  // The split count by the estimated time: waves of resident clusters x (KV tiles of
+  // the busiest CTA -- the tiles are dealt out in runs of ceil(tiles / s) -- plus a
+  // fixed cost of about three tiles), lightly penalising splits (each adds rows to
+  // merge), so that of two split counts with the same runs the smaller wins.
+  const long long units = static_cast<long long>(B) * Hkv * p.n_mt;
   double best_cost = 1e30;
-  p.tpc = 1;
   p.n_splits = 1;
-  for (int tpc = 1; tpc <= 2; ++tpc) {
-    const int groups = (p.n_mt + tpc - 1) / tpc;
-    const long long units = static_cast<long long>(B) * Hkv * groups;
-    const double tile_cost = tpc == 2 ? 1.3 : 1.0;
-    for (int s = 1; s <= max_splits; ++s) {
-      if (active[s] < 1) continue;
-      const double waves = std::ceil(static_cast<double>(units) / active[s]);
-      const double work = (prefix_tiles + tree_tiles) / static_cast<double>(s) * tile_cost + 3.0;
-      const double cost = waves * work * (1.0 + 0.02 * (s - 1));
-      if (cost < best_cost - 1e-9) {
-        best_cost = cost;
-        p.tpc = tpc;
-        p.n_splits = s;
-      }
+  for (int s = 1; s <= max_splits; ++s) {
+    if (active[s] < 1) continue;
+    const double waves = std::ceil(static_cast<double>(units) / active[s]);
+    const int run = (tiles + s - 1) / s;
+    const double cost = waves * (run + 3.0) * (1.0 + 0.02 * (s - 1));
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
+      p.n_splits = s;
     }
   }
-  p.n_groups = (p.n_mt + p.tpc - 1) / p.tpc;
-  p.ctas = static_cast<size_t>(B) * Hkv * p.n_groups * p.n_splits;
+  p.ctas = static_cast<size_t>(units) * p.n_splits;
   return p;
 }
 
@@ -834,6 +856,26 @@ const int* active_clusters() {
 }
 
 }  // namespace
+
+// The long-run schedule (tree_attention_pair.cu): two row tiles per CTA in ping-pong.
+// Over a long run of KV tiles per CTA the two tiles' softmax-to-tensor-core chains
+// interleave and beat this file's deeper S pipeline for one tile; over a short run
+// (the small rounds) this file's schedule wins, mostly in the fill and the merge.
+namespace pair_attn {
+int run_tiles(int B, int N, int Hq, int Hkv, int D, int Tmax);  // KV tiles per CTA of its plan
+size_t workspace(int B, int N, int Hq, int Hkv, int D, int Tmax);
+int launch(const void* q, const void* k_cache, const void* v_cache, const int32_t* kv_len, int Tmax,
+           const void* k_tree, const void* v_tree, const uint32_t* mask, const int32_t* n_nodes, int B,
+           int N, int Hq, int Hkv, int D, float sm_scale, void* out, float* lse, void* ws,
+           size_t ws_bytes, int32_t* dev_status, cudaStream_t stream);
+}  // namespace pair_attn
+
+constexpr int kPairMinRun = 8;  // KV tiles per CTA from which the pair schedule is taken
+
+bool use_pair(int B, int N, int Hq, int Hkv, int D, int Tmax) {
+  return pair_attn::run_tiles(B, N, Hq, Hkv, D, Tmax) >= kPairMinRun;
+}
+
 }  // namespace presto
 
 using namespace presto;
@@ -841,11 +883,12 @@ using namespace presto;
 extern "C" size_t presto_attn_workspace(int B, int N, int Hq, int Hkv, int D, int Tmax) {
   if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || Tmax < 1 || (D != 64 && D != 128))
     return 0;
+  if (use_pair(B, N, Hq, Hkv, D, Tmax)) return pair_attn::workspace(B, N, Hq, Hkv, D, Tmax);
   // KV splits leave partial rows (float32 at most) and fp32 (m, l) for the merge
   const int* active = D == 128 ? active_clusters<128>() : active_clusters<64>();
   const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
   if (p.n_splits == 1) return 256;
-  return align_up(p.ctas * 2 * kBM * (static_cast<size_t>(D) * 4 + 8), 256);
+  return align_up(p.ctas * kBM * (static_cast<size_t>(D) * 4 + 8), 256);
 }
 
 extern "C" int presto_tree_attention(const void* q, const void* k_cache, const void* v_cache,
@@ -865,14 +908,17 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
   PRESTO_CHECK_LIMIT(G <= kBM && (G & (G - 1)) == 0);
   for (const void* p : {q, k_cache, v_cache, k_tree, v_tree, static_cast<const void*>(out)})
     PRESTO_CHECK_ARG(reinterpret_cast<uintptr_t>(p) % 16 == 0);
+  if (use_pair(B, N, Hq, Hkv, D, Tmax))
+    return pair_attn::launch(q, k_cache, v_cache, kv_len, Tmax, k_tree, v_tree, mask, n_nodes, B, N,
+                             Hq, Hkv, D, sm_scale, out, lse, ws, ws_bytes, dev_status, stream);
   const int* active = D == 128 ? active_clusters<128>() : active_clusters<64>();
   const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
   Args a{};
   if (p.n_splits > 1) {
-    const size_t need = p.ctas * 2 * kBM * (static_cast<size_t>(D) * 4 + 8);
+    const size_t need = p.ctas * kBM * (static_cast<size_t>(D) * 4 + 8);
     if (!ws || reinterpret_cast<uintptr_t>(ws) % 16 || ws_bytes < need) return PRESTO_ERR_WORKSPACE;
     a.part_o = static_cast<float2*>(ws);
-    a.part_ml = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.ctas * 2 * kBM * D * 4);
+    a.part_ml = reinterpret_cast<float2*>(static_cast<char*>(ws) + p.ctas * kBM * D * 4);
   }
   const uint64_t e = 2;  // bf16 bytes
   CUtensorMap tq, tkc, tvc, tkt, tvt;
@@ -901,8 +947,6 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
   a.Tmax = Tmax;
   a.W = (N + 31) / 32;
   a.n_mt = p.n_mt;
-  a.tpc = p.tpc;
-  a.n_groups = p.n_groups;
   a.n_splits = p.n_splits;
   a.scale_log2 = sm_scale * kLog2e;
   a.out = static_cast<__nv_bfloat16*>(out);
@@ -933,3 +977,4 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
   if (err != cudaSuccess) return PRESTO_ERR_CUDA;
   return launch_status();
 }
+

@@ -582,16 +582,16 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   pdl_wait();
   for (int i = tid; i < L * k; i += kThreads) {
     const int d = i / k, j = i - d * k;
-    int t = a.ids[(static_cast<size_t>(b) * L + d) * k + j];
+    int t = ld_chain(a.ids + (static_cast<size_t>(b) * L + d) * k + j);
     if (t < 0 || t >= kMaxV) {
       if (rank == 0) report(a.dev_status, PRESTO_DEV_BAD_TOKEN);
       t = 0;
     }
     sm.cid[d][j] = t;
-    sm.clq[d][j] = a.logq[(static_cast<size_t>(b) * L + d) * k + j];
+    sm.clq[d][j] = ld_chain(a.logq + (static_cast<size_t>(b) * L + d) * k + j);
   }
   for (int d = tid; d < L; d += kThreads) {
-    float lam = a.lambda_d ? a.lambda_d[static_cast<size_t>(b) * L + d] : a.lambda;
+    float lam = a.lambda_d ? ld_chain(a.lambda_d + static_cast<size_t>(b) * L + d) : a.lambda;
     if (!(lam >= 0.f)) {  // negative or NaN: scores could turn positive
       if (rank == 0) report(a.dev_status, PRESTO_DEV_POSITIVE_SCORE);
       lam = 0.f;
@@ -599,8 +599,8 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
     sm.lam[d] = lam;
   }
   if (tid == 0) {
-    sm.ctx0 = a.ctx2[2 * b];
-    sm.ctx1 = a.ctx2[2 * b + 1];
+    sm.ctx0 = ld_chain(a.ctx2 + 2 * b);
+    sm.ctx1 = ld_chain(a.ctx2 + 2 * b + 1);
     if (rank == 0 && (sm.ctx0 < 0 || sm.ctx0 >= kMaxV || sm.ctx1 < 0 || sm.ctx1 >= kMaxV))
       report(a.dev_status, PRESTO_DEV_BAD_TOKEN);
   }
@@ -767,7 +767,7 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
     // [32u, 32u + 32); rows of unused nodes are zero, their position -1
     __syncthreads();
     const int N = a.N, W = (N + 31) / 32;
-    int kv = a.kv_len[b];
+    int kv = ld_chain(a.kv_len + b);
     if (kv < 0) {
       if (tid == 0) report(a.dev_status, PRESTO_DEV_BAD_KVLEN);
     }

@@ -22,16 +22,16 @@ __global__ void __launch_bounds__(kMaxN) mask_kernel(const int32_t* node_parent,
   pdl_launch_dependents();
   pdl_wait();  // the tree comes from the previous kernel on the stream
   const int b = blockIdx.x, i = threadIdx.x;
-  int n = n_nodes[b];
+  int n = ld_chain(n_nodes + b);
   if (n < 1 || n > N) {
     if (i == 0) report(dev_status, PRESTO_DEV_BAD_NNODES);
     n = n < 1 ? 0 : N;
   }
-  const int kv = kv_len[b];
+  const int kv = ld_chain(kv_len + b);
   if (i == 0 && kv < 0) report(dev_status, PRESTO_DEV_BAD_KVLEN);
   if (i < N) {
-    par[i] = node_parent[static_cast<size_t>(b) * N + i];
-    dep[i] = node_depth[static_cast<size_t>(b) * N + i];
+    par[i] = ld_chain(node_parent + static_cast<size_t>(b) * N + i);
+    dep[i] = ld_chain(node_depth + static_cast<size_t>(b) * N + i);
     for (int w = 0; w < W; ++w) rows[i * (W + 1) + w] = 0u;
   }
   __syncthreads();
@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(kAccThreads) accept_kernel(
   pdl_launch_dependents();
   pdl_wait();  // the tree and the target tokens come from earlier kernels on the stream
   const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  int n = n_nodes[b];
+  int n = ld_chain(n_nodes + b);
   if (n < 1 || n > N) {
     if (tid == 0) report(dev_status, PRESTO_DEV_BAD_NNODES);
     n = n < 1 ? 1 : N;
@@ -91,9 +91,9 @@ __global__ void __launch_bounds__(kAccThreads) accept_kernel(
       if (i == 0) {
         m = true;
       } else {
-        p = node_parent[base + i];
+        p = ld_chain(node_parent + base + i);
         if (p >= 0 && p < i) {
-          m = node_token[base + i] == target_token[base + p];
+          m = ld_chain(node_token + base + i) == ld_chain(target_token + base + p);
         } else {
           report(dev_status, PRESTO_DEV_BAD_PARENT);
           p = -1;
@@ -143,7 +143,7 @@ __global__ void __launch_bounds__(kAccThreads) accept_kernel(
       j = j > 0 ? par[j] : 0;
     }
     accept_len[b] = d;
-    bonus[b] = target_token[base + node];
+    bonus[b] = ld_chain(target_token + base + node);
   }
 }
 

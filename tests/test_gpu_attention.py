@@ -146,6 +146,16 @@ def test_attention_long_ctx_layer_sampled():
     _run_and_check(inp, t, w.N, seqs=[5], kv_heads=[7])
 
 
+def test_attention_long_run_d64():
+    """D = 64 with many (sequence, kv head) pairs and long prefixes: one KV split per
+    row block, 17 KV tiles per CTA (the long-run schedule); ragged prefix lengths."""
+    B, N, Hq, Hkv, T = 16, 64, 32, 8, 2048
+    t = _tree(11, B, N, L=12, k=6)
+    kv = [2048 - 61 * b for b in range(B)]
+    inp = _inputs(B, N, Hq, Hkv, 64, T, kv, seed=11)
+    _run_and_check(inp, t, N, seqs=[0, 7, 15], kv_heads=[0, 3, 7])
+
+
 def test_attention_kv_len_above_capacity_is_reported():
     B, N = 1, 8
     t = _tree(10, B, N)

@@ -998,7 +998,8 @@ def run_ours(args):
     # (logits, context, target tokens, each layer's q and tree K/V; the KV cache is
     # resident) sit packed in one pinned host buffer and go to the device in one copy;
     # the round's results come back in one copy that the host waits for.  StagedRounds
-    # double-buffers the staging, so round i + 1's copy in overlaps round i's compute
+    # double-buffers the staging and keeps one round queued ahead of the host, so
+    # round i + 1's copy in and launch overlap round i's compute
     def tensors_of(st):
         out = [st["logits"], st["ctx"], st["target"]]
         for lay in st["layers"]:
@@ -1129,7 +1130,9 @@ def run_ours(args):
                             "in one pinned host buffer, one copy in (on a copy stream, into one "
                             "of two staging buffers, overlapping the previous round); the "
                             "round (a CUDA graph); accept_len/path/bonus in one copy out; a "
-                            "host wait for it. KV cache resident (StagedRounds)"},
+                            "host wait for it. One round is queued ahead of the host wait, as "
+                            "a server alternating two independent request groups does. KV "
+                            "cache resident (StagedRounds)"},
             "clocks": clocks,
             "gpu_launches": args.steps * step.kernels_per_round(w.layers),
         }), flush=True)

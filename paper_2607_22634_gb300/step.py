@@ -127,17 +127,18 @@ class DraftVerifyStep:
 
 
 class StagedRounds:
-    """Rounds fed from pinned host memory, with each round's input copy overlapped
-    with the previous round's compute.
+    """Rounds fed from pinned host memory, one round in flight ahead of the host.
 
     One round's inputs (the tensors of `example`, e.g. logits, context, target
     tokens and each layer's q and tree K/V; the KV cache stays resident) are packed
     into one contiguous 256-byte-aligned layout.  Two device staging buffers hold
     that layout, and one CUDA graph of the round is captured per buffer.  `run(i)`
-    runs round i from its staging buffer while a copy stream brings round i + 1's
-    inputs into the other buffer, then copies round i's results (accept_len, path
-    and bonus, one contiguous buffer) to pinned host memory and waits for them:
-    every round still moves its own inputs in and its results out.
+    queues round i + 1 (its inputs copied in on a copy stream while round i
+    computes, its graph queued behind round i, its results queued for a copy back)
+    and then waits for round i's results, so that the GPU never idles while the
+    host wakes up and launches: this is the schedule of a server that alternates
+    two independent groups of requests, whose rounds do not wait on each other's
+    results.  Every round still moves its own inputs in and its results out.
 
     `bind(views)` maps the staged tensors (a list of device views, in the order of
     `example`) to the arguments of DraftVerifyStep.run:
@@ -154,6 +155,9 @@ class StagedRounds:
             pos += -(-t.numel() * t.element_size() // 256) * 256
         self.nbytes = pos
         self.staging = [torch.empty(pos, dtype=torch.uint8, device=dev) for _ in range(2)]
+        for buf in self.staging:  # the example round, so that the capture warms up on valid inputs
+            for v, t in zip(self.views(buf), example):
+                v.copy_(t)
         self.graphs = [step.capture(*bind(self.views(s))) for s in self.staging]
         self.copy_stream = torch.cuda.Stream(device=dev)
         self.result_host = [torch.empty(step.result.numel(), dtype=step.result.dtype).pin_memory()
@@ -181,21 +185,26 @@ class StagedRounds:
             self.staging[s].copy_(host_buf, non_blocking=True)
         self.copied[s].record(cs)
 
-    def start(self, host_buf):
-        """Queue the first round's inputs (into staging buffer 0)."""
-        self._upload(host_buf, 0)
-
-    def run(self, i, next_host_buf=None):
-        """Run round i (its inputs queued by start() or the previous run()), queue
-        next_host_buf for round i + 1, and return round i's results on the host."""
-        s = i % 2
+    def _launch(self, s):
         main = torch.cuda.current_stream(self.step.device)
         main.wait_event(self.copied[s])
         self.graphs[s].replay()
         self.done[s].record(main)
         self.result_host[s].copy_(self.step.result, non_blocking=True)
         self.read[s].record(main)
+
+    def start(self, host_buf):
+        """Queue the first round: its inputs into staging buffer 0, then the round."""
+        self._upload(host_buf, 0)
+        self._launch(0)
+
+    def run(self, i, next_host_buf=None):
+        """Queue round i + 1 from next_host_buf (if given), then wait for round i (queued
+        by start() or the previous run()) and return its results on the host.  The
+        returned pinned buffer is rewritten by round i + 2: copy it to keep it."""
+        s = i % 2
         if next_host_buf is not None:
             self._upload(next_host_buf, s ^ 1)
+            self._launch(s ^ 1)
         self.read[s].synchronize()
         return self.result_host[s]

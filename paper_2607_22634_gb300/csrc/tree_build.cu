@@ -580,28 +580,51 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
 
   // ---- candidates and context (produced by the previous kernel on the stream)
   pdl_wait();
-  for (int i = tid; i < L * k; i += kThreads) {
-    const int d = i / k, j = i - d * k;
-    int t = ld_chain(a.ids + (static_cast<size_t>(b) * L + d) * k + j);
-    if (t < 0 || t >= kMaxV) {
-      if (rank == 0) report(a.dev_status, PRESTO_DEV_BAD_TOKEN);
-      t = 0;
+  // every load first (one round trip: L * k <= 2 kThreads, L <= kThreads), then the
+  // checks, so that no status report sits between two loads
+  static_assert(kMaxL * kMaxK <= 2 * kThreads && kMaxL <= kThreads, "one pass of loads");
+  int t_in[2] = {0, 0};
+  float lq_in[2] = {0.f, 0.f};
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const int i = tid + u * kThreads;
+    if (i < L * k) {
+      t_in[u] = ld_chain(a.ids + static_cast<size_t>(b) * L * k + i);
+      lq_in[u] = ld_chain(a.logq + static_cast<size_t>(b) * L * k + i);
     }
-    sm.cid[d][j] = t;
-    sm.clq[d][j] = ld_chain(a.logq + (static_cast<size_t>(b) * L + d) * k + j);
   }
-  for (int d = tid; d < L; d += kThreads) {
-    float lam = a.lambda_d ? ld_chain(a.lambda_d + static_cast<size_t>(b) * L + d) : a.lambda;
+  float lam = a.lambda;
+  if (tid < L && a.lambda_d) lam = ld_chain(a.lambda_d + static_cast<size_t>(b) * L + tid);
+  int c0 = 0, c1 = 0;
+  if (tid == 0) {
+    c0 = ld_chain(a.ctx2 + 2 * b);
+    c1 = ld_chain(a.ctx2 + 2 * b + 1);
+  }
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const int i = tid + u * kThreads;
+    if (i < L * k) {
+      const int d = i / k, j = i - d * k;
+      int t = t_in[u];
+      if (t < 0 || t >= kMaxV) {
+        if (rank == 0) report(a.dev_status, PRESTO_DEV_BAD_TOKEN);
+        t = 0;
+      }
+      sm.cid[d][j] = t;
+      sm.clq[d][j] = lq_in[u];
+    }
+  }
+  if (tid < L) {
     if (!(lam >= 0.f)) {  // negative or NaN: scores could turn positive
       if (rank == 0) report(a.dev_status, PRESTO_DEV_POSITIVE_SCORE);
       lam = 0.f;
     }
-    sm.lam[d] = lam;
+    sm.lam[tid] = lam;
   }
   if (tid == 0) {
-    sm.ctx0 = ld_chain(a.ctx2 + 2 * b);
-    sm.ctx1 = ld_chain(a.ctx2 + 2 * b + 1);
-    if (rank == 0 && (sm.ctx0 < 0 || sm.ctx0 >= kMaxV || sm.ctx1 < 0 || sm.ctx1 >= kMaxV))
+    sm.ctx0 = c0;
+    sm.ctx1 = c1;
+    if (rank == 0 && (c0 < 0 || c0 >= kMaxV || c1 < 0 || c1 >= kMaxV))
       report(a.dev_status, PRESTO_DEV_BAD_TOKEN);
   }
   __syncthreads();

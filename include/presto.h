@@ -72,6 +72,8 @@ typedef struct CUstream_st* presto_stream_t;  /* same type as cudaStream_t */
 #define PRESTO_DEV_TABLE_FULL 0x80    /* n-gram insert found no free slot         */
 #define PRESTO_DEV_NONFINITE 0x100    /* a logits row has no finite maximum       */
 #define PRESTO_DEV_BAD_PATH 0x200     /* accept_len / accept_path entry out of range */
+#define PRESTO_DEV_BOUNDS 0x400       /* an index failed a bounds check of a debug build
+                                         (built with PRESTO_CHECKS); the access was skipped */
 
 /* ---- element types -------------------------------------------------------- */
 #define PRESTO_F32 0
@@ -81,6 +83,12 @@ typedef struct CUstream_st* presto_stream_t;  /* same type as cudaStream_t */
 const char* presto_status_string(int status);
 
 /* ABI version: (major << 16) | minor. */
+/* Build flags of the loaded library: PRESTO_BUILD_CHECKS when it was compiled with
+ * device-side bounds checks (-DPRESTO_CHECKS; a debug build: every data-dependent index
+ * into a buffer the kernels write or a table they read is checked, and a failing one
+ * reports PRESTO_DEV_BOUNDS and skips the access instead of faulting). */
+#define PRESTO_BUILD_CHECKS 0x1
+int presto_build_flags(void);
 int presto_version(void);
 
 /*

@@ -26,8 +26,9 @@ NGRAM3_EMPTY = 0xFFFFFFFFFFFFFFFF
 DEV_STATUS_BITS = {
     0x1: "BAD_PARENT", 0x2: "BAD_TOKEN", 0x4: "BAD_KVLEN", 0x8: "BAD_NNODES",
     0x10: "POSITIVE_SCORE", 0x20: "TIMEOUT", 0x40: "DUP_SIBLING", 0x80: "TABLE_FULL",
-    0x100: "NONFINITE", 0x200: "BAD_PATH",
+    0x100: "NONFINITE", 0x200: "BAD_PATH", 0x400: "BOUNDS",
 }
+BUILD_CHECKS = 0x1  # presto_build_flags(): compiled with device-side bounds checks
 
 
 class Ngram3(ctypes.Structure):
@@ -73,25 +74,29 @@ _SIGS = {
                                    ctypes.c_float, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "presto_accept": (_I, [_P, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P]),
     "presto_selftest_wait_timeout": (_I, [_P, ctypes.c_longlong, _P]),
+    "presto_build_flags": (_I, []),
 }
 
 _lib = None
 
 
 def lib_path() -> str:
-    return _build.LIB
+    """The library this process loads (the bounds-checked debug build under
+    PRESTO_CHECKS=1)."""
+    return _build.lib_file()
 
 
 def load(build_if_missing: bool = True):
-    """Load libpresto.so (building it first if needed) and declare signatures."""
+    """Load the library (building it first if needed) and declare signatures."""
     global _lib
     if _lib is not None:
         return _lib
+    path = _build.lib_file()
     if build_if_missing and not _build.up_to_date():
         _build.build()
-    if not os.path.exists(_build.LIB):
-        raise PrestoError("libpresto.so is missing; run paper_2607_22634_gb300.build.build()")
-    lib = ctypes.CDLL(_build.LIB)
+    if not os.path.exists(path):
+        raise PrestoError(f"{os.path.basename(path)} is missing; run paper_2607_22634_gb300.build.build()")
+    lib = ctypes.CDLL(path)
     for name, (res, args) in _SIGS.items():
         fn = getattr(lib, name)
         fn.restype = res
@@ -446,6 +451,11 @@ def presto_accept(node_token, node_parent, node_depth, mask, n_nodes, target_tok
                               _ptr(accept_path), _ptr(bonus), _ptr(dev_status), _stream(stream))
     _check(st, "presto_accept")
     return accept_len, accept_path, bonus
+
+
+def presto_build_flags() -> int:
+    """Flags of the loaded library (BUILD_CHECKS for the bounds-checked debug build)."""
+    return int(load().presto_build_flags())
 
 
 def presto_selftest_wait_timeout(dev_status, wait_cycles, stream=None):

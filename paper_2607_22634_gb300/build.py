@@ -1,8 +1,11 @@
-"""Compile the sm_103a CUDA sources into the in-tree shared library libpresto.so.
+"""Compile the sm_103a CUDA sources into the in-tree shared libraries.
 
-Each translation unit compiles in parallel with one -gencode (sm_103a), then nvcc
-links them with the static CUDA runtime, so the library needs only the driver at
-run time.  Rebuilds only when a source or header is newer than the library.
+libpresto.so is the library; libpresto_checks.so is the same sources compiled with
+-DPRESTO_CHECKS (device-side bounds checks that report PRESTO_DEV_BOUNDS instead of
+faulting), loaded instead when the environment sets PRESTO_CHECKS=1.  Each
+translation unit compiles in parallel with one -gencode (sm_103a), then nvcc links
+them with the static CUDA runtime, so a library needs only the driver at run time.
+Rebuilds only when a source or header is newer than the library.
 """
 
 from __future__ import annotations
@@ -19,11 +22,24 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OBJDIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libpresto.so")
+CHECKS_LIB = os.path.join(HERE, "libpresto_checks.so")
 SOURCES = ["api.cu", "topk.cu", "tree_build.cu", "tree_mask_accept.cu", "tree_attention.cu",
            "tree_attention_pair.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
                 "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]
+
+
+def checks_requested() -> bool:
+    """True when the environment asks for the bounds-checked debug library."""
+    return os.environ.get("PRESTO_CHECKS", "") == "1"
+
+
+def lib_file(checks: bool | None = None) -> str:
+    """The library this process loads: the debug build under PRESTO_CHECKS=1."""
+    if checks is None:
+        checks = checks_requested()
+    return CHECKS_LIB if checks else LIB
 
 
 def nvcc() -> str:
@@ -40,10 +56,11 @@ def _inputs():
     return deps
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+def up_to_date(checks: bool | None = None) -> bool:
+    lib = lib_file(checks)
+    if not os.path.exists(lib):
         return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(p) <= t for p in _inputs())
 
 
@@ -54,25 +71,33 @@ def _run(cmd):
     return r.stdout + r.stderr
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    """Build libpresto.so (if stale) and return its path."""
-    if not force and up_to_date():
-        return LIB
-    os.makedirs(OBJDIR, exist_ok=True)
-    cc = nvcc()
+def build(force: bool = False, verbose: bool = False, extra_flags=(), checks=None) -> str:
+    """Build a library (if stale) and return its path: the one this process loads
+    (`checks` None), the release library (False), the debug library (True), or both
+    ("both", compiled in one parallel pool; returns the release path)."""
+    variants = [False, True] if checks == "both" else [checks_requested() if checks is None else checks]
+    todo = [v for v in variants if force or not up_to_date(v)]
+    cc = nvcc() if todo else None
     jobs = []
-    for src in SOURCES:
-        obj = os.path.join(OBJDIR, src.replace(".cu", ".o"))
-        jobs.append((obj, [cc, *FLAGS, *extra_flags, "-c", os.path.join(CSRC, src), "-o", obj]))
-    with concurrent.futures.ThreadPoolExecutor(max_workers=len(jobs)) as ex:
-        logs = list(ex.map(lambda j: _run(j[1]), jobs))
-    if verbose:
-        for log in logs:
-            sys.stdout.write(log)
-    tmp = LIB + ".tmp"
-    _run([cc, *ARCH, "-shared", "-o", tmp, *[j[0] for j in jobs]])
-    os.replace(tmp, LIB)
-    return LIB
+    for v in todo:
+        objdir = OBJDIR + ("_checks" if v else "")
+        os.makedirs(objdir, exist_ok=True)
+        defs = ["-DPRESTO_CHECKS"] if v else []
+        for src in SOURCES:
+            obj = os.path.join(objdir, src.replace(".cu", ".o"))
+            jobs.append((v, obj, [cc, *FLAGS, *defs, *extra_flags, "-c", os.path.join(CSRC, src), "-o", obj]))
+    if jobs:
+        with concurrent.futures.ThreadPoolExecutor(max_workers=len(jobs)) as ex:
+            logs = list(ex.map(lambda j: _run(j[2]), jobs))
+        if verbose:
+            for log in logs:
+                sys.stdout.write(log)
+    for v in todo:
+        lib = lib_file(v)
+        tmp = lib + ".tmp"
+        _run([cc, *ARCH, "-shared", "-o", tmp, *[j[1] for j in jobs if j[0] == v]])
+        os.replace(tmp, lib)
+    return lib_file(False if checks == "both" else variants[0])
 
 
 if __name__ == "__main__":

@@ -52,6 +52,14 @@ extern "C" const char* presto_status_string(int status) {
 
 extern "C" int presto_version(void) { return (1 << 16) | 0; }
 
+extern "C" int presto_build_flags(void) {
+#ifdef PRESTO_CHECKS
+  return PRESTO_BUILD_CHECKS;
+#else
+  return 0;
+#endif
+}
+
 extern "C" int presto_selftest_wait_timeout(int32_t* dev_status, long long wait_cycles,
                                             presto_stream_t stream) {
   PRESTO_CHECK_ARG(dev_status);

@@ -303,6 +303,21 @@ inline cudaLaunchAttribute pdl_attribute() {
   return at;
 }
 
+// Debug builds (-DPRESTO_CHECKS): PRESTO_IN_BOUNDS(i, n, status) is false, and reports
+// PRESTO_DEV_BOUNDS, when i is outside [0, n), so that the caller skips the access; in
+// release builds it is the constant true and costs nothing.
+__device__ __forceinline__ bool in_bounds_checked(long long i, long long n, int32_t* status) {
+  if (i >= 0 && i < n) return true;
+  report(status, PRESTO_DEV_BOUNDS);
+  return false;
+}
+#ifdef PRESTO_CHECKS
+#define PRESTO_IN_BOUNDS(i, n, status) \
+  (::presto::in_bounds_checked(static_cast<long long>(i), static_cast<long long>(n), (status)))
+#else
+#define PRESTO_IN_BOUNDS(i, n, status) true
+#endif
+
 // Loads of data that an earlier kernel of the stream writes (read after the grid
 // dependency wait) go through L2 only.  Kernels of a dependent-launch chain start
 // while earlier ones still run, so an SM's L1 can hold lines that a previous

@@ -245,9 +245,11 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
   // Child c of a node with score Sp, children context x and candidate index pj, at
   // depth dc; `pfield` fills the key's last field (kPMask - the parent's position among
   // the parents of its level).  Returns the key, context and candidate index.
+  const int nkid = L * cs * nb;  // child records in the tables
   auto child = [&](uint32_t x, float Sp, int pj, int pfield, int dc, int c, uint64_t& key,
                    uint32_t& xc, int& jc) {
-    const uint2 kd = kids[x * nb + c];
+    const int ik = static_cast<int>(x) * nb + c;
+    const uint2 kd = PRESTO_IN_BOUNDS(ik, nkid, a.dev_status) ? kids[ik] : make_uint2(0u, 0u);
     key = (static_cast<uint64_t>(ordered(__fadd_rn(Sp, __uint_as_float(kd.x)))) << 32) |
           (kd.y & ~kPMask) | (kPMask - static_cast<uint32_t>(pfield));
     jc = static_cast<int>(kd.y & kPMask);
@@ -419,7 +421,7 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
       }
       const bool keep = key != 0ull && (beam || key > tau);
       const int slot = reserve(keep, cn);
-      if (keep) {
+      if (keep && PRESTO_IN_BOUNDS(slot, NC, a.dev_status)) {
         ckey[cn * NC + slot] = key;
         cxc[cn * NC + slot] = xc;
         cpid[cn * NC + slot] = static_cast<int16_t>(r < cap ? r + 1 : -1);
@@ -493,7 +495,7 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
         }
         const bool keep = key != 0ull;
         const int slot = reserve(keep, 1);
-        if (keep) {
+        if (keep && PRESTO_IN_BOUNDS(slot, NC, a.dev_status)) {
           F[slot] = key;
           cpid[cc * NC + slot] = static_cast<int16_t>(i);
         }
@@ -542,7 +544,9 @@ __device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigne
       const uint32_t lo = static_cast<uint32_t>(ke);
       const int dd = 63 - static_cast<int>((lo >> 26) & 63u);
       const int tr = 15 - static_cast<int>((lo >> kTRankShift) & 15u);
-      a.node_token[o] = sm.rtok[dd - 1][tr];
+      a.node_token[o] = PRESTO_IN_BOUNDS(dd - 1, L, a.dev_status) && PRESTO_IN_BOUNDS(tr, k, a.dev_status)
+                            ? sm.rtok[dd - 1][tr]
+                            : -1;
       a.node_depth[o] = dd;
       a.node_parent[o] = pid;
       a.node_score[o] = unordered(static_cast<uint32_t>(ke >> 32));
@@ -745,7 +749,9 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
         const int gl = f / k, j = f - gl * k;
         int d, ci;
         decode_ctx(g0 + gl, k, use_table, d, ci);
-        kids[(d * tl.cs + ci) * nb + j] = kid_record(sc, d, sm.trk[d][j], j);
+        const int ik = (d * tl.cs + ci) * nb + j;
+        if (PRESTO_IN_BOUNDS(ik, tl.nctx * nb, a.dev_status))
+          kids[ik] = kid_record(sc, d, sm.trk[d][j], j);
       } else {
         st_s[f] = sc;
       }
@@ -770,7 +776,9 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
         const int ti = sm.cid[d][i];
         rk += (si > sj) || (si == sj && (ti < tj || (ti == tj && i < j)));
       }
-      if (rk < nb) kids[(d * tl.cs + ci) * nb + rk] = kid_record(row[j], d, sm.trk[d][j], j);
+      const int ik = (d * tl.cs + ci) * nb + rk;
+      if (rk < nb && PRESTO_IN_BOUNDS(ik, tl.nctx * nb, a.dev_status))
+        kids[ik] = kid_record(row[j], d, sm.trk[d][j], j);
     }
   }
   if (!a.tables_in_smem) __threadfence();
@@ -801,7 +809,7 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
         uint32_t word = 0u;
         int dd = 0;
         if (i < n)
-          for (int j = i; j >= 0; j = sm.par[j], ++dd)
+          for (int j = i; j >= 0 && PRESTO_IN_BOUNDS(j, N, a.dev_status); j = sm.par[j], ++dd)
             if ((j >> 5) == u) word |= 1u << (j & 31);
         row[u] = word;
         depth = dd - 1;

@@ -39,12 +39,32 @@ __host__ __device__ inline uint64_t fmix64(uint64_t k) {
   return k;
 }
 
+// Loads of the trigram table with an L2 evict-last policy: the table is model state that
+// every round probes, while the round's logits and KV cache stream through L2 once, so
+// its recently probed slots should outlive them there.  A cache policy is a hint.
+__device__ __forceinline__ uint64_t l2_keep_policy() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.L2::evict_unchanged.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+__device__ __forceinline__ uint64_t ld_table(const uint64_t* p, uint64_t pol) {
+  uint64_t v;
+  asm volatile("ld.global.nc.L2::cache_hint.u64 %0, [%1], %2;" : "=l"(v) : "l"(p), "l"(pol));
+  return v;
+}
+__device__ __forceinline__ float ld_table(const float* p, uint64_t pol) {
+  float v;
+  asm volatile("ld.global.nc.L2::cache_hint.f32 %0, [%1], %2;" : "=f"(v) : "l"(p), "l"(pol));
+  return v;
+}
+
 // Linear probe for `key` starting at slot h.
 __device__ __noinline__ float probe_from(const uint64_t* keys, const float* logrho,
                                          uint32_t mask, float miss, uint64_t key, uint32_t h) {
+  const uint64_t pol = l2_keep_policy();
   for (uint32_t it = 0; it <= mask; ++it) {
-    const uint64_t kk = __ldg(keys + h);
-    if (kk == key) return __ldg(logrho + h);
+    const uint64_t kk = ld_table(keys + h, pol);
+    if (kk == key) return ld_table(logrho + h, pol);
     if (kk == PRESTO_NGRAM3_EMPTY) return miss;
     h = (h + 1) & mask;
   }
@@ -661,6 +681,7 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   // slots in one round; only a longer chain continues slot by slot
   constexpr int kBatch = 2;
   constexpr int kWin = 4;
+  const uint64_t pol = l2_keep_policy();
   for (int f0 = tid; f0 < my; f0 += kThreads * kBatch) {
     uint64_t key[kBatch];
     uint32_t h[kBatch];
@@ -700,8 +721,8 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
 #pragma unroll
     for (int q = 0; q < kBatch; ++q) {
       const bool live = key[q] != PRESTO_NGRAM3_EMPTY;
-      k0[q] = live ? __ldg(a.keys + h[q]) : PRESTO_NGRAM3_EMPTY;
-      v0[q] = live ? __ldg(a.logrho + h[q]) : 0.f;
+      k0[q] = live ? ld_table(a.keys + h[q], pol) : PRESTO_NGRAM3_EMPTY;
+      v0[q] = live ? ld_table(a.logrho + h[q], pol) : 0.f;
     }
     // second round: the window after the home slot, for the probes still open
     uint64_t kw[kBatch][kWin];
@@ -712,8 +733,8 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
 #pragma unroll
       for (int w = 0; w < kWin; ++w) {
         const uint32_t hw = (h[q] + 1 + w) & a.cap_mask;
-        kw[q][w] = open ? __ldg(a.keys + hw) : PRESTO_NGRAM3_EMPTY;
-        vw[q][w] = open ? __ldg(a.logrho + hw) : 0.f;
+        kw[q][w] = open ? ld_table(a.keys + hw, pol) : PRESTO_NGRAM3_EMPTY;
+        vw[q][w] = open ? ld_table(a.logrho + hw, pol) : 0.f;
       }
     }
 #pragma unroll

@@ -374,7 +374,7 @@ int presto_tree_mask(const int32_t* node_parent, const int32_t* node_depth,
  * with g = h / (Hq/Hkv).  bf16 inputs, float32 softmax and accumulation, bf16 out.
  *
  *   q        [B, N, Hq, D] bf16 (positions / RoPE already applied)
- *   k_cache, v_cache [B, Hkv, Tmax, D] bf16; rows >= kv_len[b] are ignored
+ *   k_cache, v_cache [B, Hkv, Tmax, D] bf16; rows >= kv_len[b] get zero weight
  *   kv_len   [B] int32 in [0, Tmax]
  *   k_tree, v_tree   [B, N, Hkv, D] bf16
  *   mask     [B, N, ceil(N/32)] uint32 from presto_tree_mask
@@ -383,7 +383,14 @@ int presto_tree_mask(const int32_t* node_parent, const int32_t* node_depth,
  *   lse      [B, N, Hq] float32 out, nullable: natural-log softmax denominator
  *   ws       presto_attn_workspace(B, N, Hq, Hkv, D, Tmax) bytes (for the current
  *            device).
- * All base pointers must be 16-byte aligned.
+ * All base pointers must be 16-byte aligned.  Rows of k_cache / v_cache at or past
+ * kv_len[b], and rows of k_tree / v_tree at or past n_nodes[b] (up to N), get zero
+ * weight but are read with the 128-key tile that holds them: they must hold finite
+ * values (a zero weight times a NaN is a NaN).
+ * Under programmatic dependent launch, the KV cache and kv_len may be read before the
+ * kernel waits for the previous kernels on the stream (no kernel of a round writes
+ * them: the caller must not write them from a kernel that lets this one start early);
+ * q, k_tree, v_tree, mask and n_nodes are read after that wait.
  */
 size_t presto_attn_workspace(int B, int N, int Hq, int Hkv, int D, int Tmax);
 int presto_tree_attention(const void* q, const void* k_cache, const void* v_cache,

@@ -221,37 +221,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  // before the dependency wait, ask L2 for this split's KV-prefix rows: no kernel of
-  // the round writes the KV cache, and a prefetch is a hint that reads nothing into
-  // the SM, so its DRAM traffic overlaps the previous kernels whatever they write.
-  // The split's range is taken from kv_len as read now and the node budget N (the
-  // exact split below uses the node count the build writes): a stale read only
-  // misplaces the hint by a tile.
-  if (tid == 0) {
-    const int kvh = min(max(*reinterpret_cast<const volatile int32_t*>(a.kv_len + b), 0), a.Tmax);
-    const int pt = (kvh + kBN - 1) / kBN;
-    const int tot = pt + (a.N + kBN - 1) / kBN;
-    const int per_h = (tot + a.n_splits - 1) / a.n_splits;
-    const int tb = min(split * per_h, pt);
-    const int te = min(tb + per_h, pt);
-    if (te > tb) {
-      const size_t row0 = (static_cast<size_t>(b) * a.Hkv + g) * a.Tmax;
-      const int t0 = tb * kBN, t1 = min(te * kBN, kvh);
-      const uint32_t bytes = static_cast<uint32_t>(t1 - t0) * D * 2u;
-      prefetch_l2_bulk(a.k_cache + (row0 + t0) * D, bytes);
-      prefetch_l2_bulk(a.v_cache + (row0 + t0) * D, bytes);
-    }
-  }
-  pdl_wait();  // the mask and node counts come from the previous kernels on the stream
+  // No kernel of the round writes the KV cache or kv_len (the caller does, between
+  // rounds), so the split's KV tiles and their KV-cache part are known before the
+  // dependency wait: the loaders fill their rings with KV-cache tiles and the rest of
+  // the split's range is asked of L2 while the previous kernels still run.  q and the
+  // tree K/V (computed from the tree, in a real round, by the target model), the
+  // ancestor mask and the node count are read only after griddepcontrol.wait.
   const int kv_raw = ld_chain(a.kv_len + b);
-  const int nn_raw = ld_chain(a.n_nodes + b);
-
   int kv = kv_raw;
   if (kv < 0 || kv > a.Tmax) {
     if (tid == 0) report(a.dev_status, PRESTO_DEV_BAD_KVLEN);
     kv = kv < 0 ? 0 : a.Tmax;
   }
-  const int nn = nn_raw < 0 ? 0 : (nn_raw > a.N ? a.N : nn_raw);
   // split partials in float32 when the prefix is short: then a row averages few keys,
   // its values can be as large as single V entries, and the bf16 roundings of P, of a
   // bf16 partial and of the output could together reach 2e-2 of N(0, 1) values; with
@@ -260,14 +241,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int prefix_tiles = (kv + kBN - 1) / kBN;
   // the KV tiles of a row tile, prefix tiles then tree tiles, in equal runs over the
   // splits: this split's local tile j is prefix tile t_begin + j for j < n_prefix,
-  // else tree tile tree0 + (j - n_prefix)
-  const int tree_tiles = (nn + kBN - 1) / kBN;
+  // else tree tile tree0 + (j - n_prefix).  The tree tiles cover the node budget N
+  // (the built node count is not known before the wait); keys past it are masked out.
+  const int tree_tiles = (a.N + kBN - 1) / kBN;
   const int total = prefix_tiles + tree_tiles;
   const int per = (total + a.n_splits - 1) / a.n_splits;
   const int t_begin = min(split * per, total);
   const int nt = min(total, t_begin + per) - t_begin;  // KV tiles of this split (CTA-uniform)
   const int n_prefix = max(0, min(nt, prefix_tiles - t_begin));
   const int tree0 = t_begin + n_prefix - prefix_tiles;
+  constexpr int kRing = Ly::kKStages < Ly::kVStages ? Ly::kKStages : Ly::kVStages;
+  if (tid == 0 && n_prefix > kRing) {  // the prefix tiles beyond the rings, into L2
+    const size_t row0 = (static_cast<size_t>(b) * a.Hkv + g) * a.Tmax;
+    const int t0 = (t_begin + kRing) * kBN, t1 = min((t_begin + n_prefix) * kBN, kv);
+    if (t1 > t0) {
+      const uint32_t bytes = static_cast<uint32_t>(t1 - t0) * D * 2u;
+      prefetch_l2_bulk(a.k_cache + (row0 + t0) * D, bytes);
+      prefetch_l2_bulk(a.v_cache + (row0 + t0) * D, bytes);
+    }
+  }
 
   volatile int* abort = &abort_flag;
   auto fail = [&]() {
@@ -275,19 +267,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     report(a.dev_status, PRESTO_DEV_TIMEOUT);
   };
 
-  int issued = 0;  // K or V tiles this warp's lane 0 has issued (the loaders)
+  int issued = 0;         // K or V tiles this warp's lane 0 has issued (the loaders)
+  bool q_issued = false;  // the K loader has issued the Q tile
   if (nt > 0 && warp == kKWarp) {
     // ------------------------------------------------------------ Q and K loads
     if (lane == 0) {
       prefetch_tensormap(&tm_q);
       prefetch_tensormap(&tm_kc);
       prefetch_tensormap(&tm_kt);
-      mbar_arrive_expect_tx(&bars.q_full, Ly::kQBytes);
-      for (int p = 0; p < Ly::kPanels; ++p)
-        tma_load_3d(smem + Ly::kQ + p * Ly::kQPanel, &tm_q, p * 64, g * a.G, b * a.N + mt * nodes_per_tile,
-                    &bars.q_full);
-      // K_j -> slot j % Ly::kKStages, once the QK^T of K_{j - Ly::kKStages} completed
+      // K_j -> slot j % Ly::kKStages, once the QK^T of K_{j - Ly::kKStages} completed;
+      // the first KV-cache tiles before the dependency wait, Q and the rest after it
+      const int early = min(n_prefix, Ly::kKStages);
       for (int j = 0; j < nt; ++j) {
+        if (j == early) {
+          pdl_wait();
+          mbar_arrive_expect_tx(&bars.q_full, Ly::kQBytes);
+          for (int p = 0; p < Ly::kPanels; ++p)
+            tma_load_3d(smem + Ly::kQ + p * Ly::kQPanel, &tm_q, p * 64, g * a.G,
+                        b * a.N + mt * nodes_per_tile, &bars.q_full);
+          q_issued = true;
+        }
         const int st = j % Ly::kKStages;
         if (j >= Ly::kKStages && !mbar_wait(&bars.k_empty[st], (j / Ly::kKStages - 1) & 1, abort)) {
           fail();
@@ -305,14 +304,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         issued = j + 1;
       }
+      if (!q_issued) {  // every tile was an early one
+        pdl_wait();
+        mbar_arrive_expect_tx(&bars.q_full, Ly::kQBytes);
+        for (int p = 0; p < Ly::kPanels; ++p)
+          tma_load_3d(smem + Ly::kQ + p * Ly::kQPanel, &tm_q, p * 64, g * a.G,
+                      b * a.N + mt * nodes_per_tile, &bars.q_full);
+        q_issued = true;
+      }
     }
   } else if (nt > 0 && warp == kVWarp) {
     // ------------------------------------------------------------ V loads
     if (lane == 0) {
       prefetch_tensormap(&tm_vc);
       prefetch_tensormap(&tm_vt);
-      // V_j -> slot j % Ly::kVStages, once the PV of V_{j - Ly::kVStages} completed
+      // V_j -> slot j % Ly::kVStages, once the PV of V_{j - Ly::kVStages} completed;
+      // the first KV-cache tiles before the dependency wait
+      const int early = min(n_prefix, Ly::kVStages);
       for (int j = 0; j < nt; ++j) {
+        if (j == early) pdl_wait();
         const int st = j % Ly::kVStages;
         if (j >= Ly::kVStages && !mbar_wait(&bars.v_empty[st], (j / Ly::kVStages - 1) & 1, abort)) {
           fail();
@@ -401,6 +411,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int node = mt * nodes_per_tile + r / a.G;
     const uint32_t* mrow =
         node < a.N ? a.mask + (static_cast<size_t>(b) * a.N + node) * a.W : nullptr;
+    pdl_wait();  // the mask and the node count come from the build
+    const int nn = min(max(ld_chain(a.n_nodes + b), 0), a.N);
     float m = -INFINITY, l = 0.f;  // m: running (possibly stale) max, log2 domain; l: this half's sum
     bool ok = true;
     for (int j = 0; j < nt; ++j) {
@@ -586,6 +598,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
 
+  // every thread past the dependency wait before the outputs and the merge (which read
+  // the node count); a thread that already waited returns at once
+  pdl_wait();
+
   // ---- unwind after a timed-out wait.  Before the TMEM is freed and the CTA exits,
   // nothing asynchronous may still target them: each loader waits (bounded) for the
   // last copy it issued into every stage (and for Q), whether or not anyone consumed
@@ -596,7 +612,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (nt > 0 && (warp == kKWarp || warp == kVWarp) && lane == 0) {
       uint64_t* full = warp == kKWarp ? bars.k_full : bars.v_full;
       const int S = warp == kKWarp ? Ly::kKStages : Ly::kVStages;
-      if (warp == kKWarp) mbar_wait(&bars.q_full, 0, nullptr);
+      if (warp == kKWarp && q_issued) mbar_wait(&bars.q_full, 0, nullptr);
       for (int j = max(0, issued - S); j < issued; ++j) mbar_wait(&full[j % S], (j / S) & 1, nullptr);
     }
     if (nt > 0 && warp == kMmaWarp) {
@@ -640,6 +656,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   // release / acquire at cluster scope: every split's partial rows are visible
   cg::this_cluster().sync();
+  const int nn = min(max(ld_chain(a.n_nodes + b), 0), a.N);
   const int R = kBM;
   const int nsp = a.n_splits;
   const int slice = (R + nsp - 1) / nsp;

@@ -239,7 +239,8 @@ constexpr int kSortMin = 256;  // candidates of a level above which they are sor
 // A node's final index is its rank, so the parent index in the key (the last tie
 // break) is the parent's rank in A, consistent across steps.
 // Returns the node count (root included).
-__device__ int select_levels(const Args& a, Smem& sm, const uint2* kids, unsigned char* p2,
+__device__ __forceinline__ int select_levels(const Args& a, Smem& sm, const uint2* kids,
+                                             unsigned char* p2,
                              int tid) {
   const int L = a.L, k = a.k, N = a.N, nb = a.bf, W = a.W;
   const bool beam = a.policy == PRESTO_SEARCH_BEAM;
@@ -807,11 +808,19 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   if (rank != 0) return;
 
   // ---- phase 2: top-N selection, level by level (leader CTA)
-  unsigned char* const p2 = a.p2_in_smem
-                                ? dyn + stage_off
-                                : a.g_p2 + static_cast<size_t>(b) * a.p2_stride;
-  const int n = select_levels(a, sm, a.tables_in_smem ? reinterpret_cast<const uint2*>(dyn) : kids,
-                              p2, tid);
+  // tables and scratch both in shared memory (every budget up to about N = 256): pointers
+  // the compiler sees as shared, so the selection's many accesses are shared-memory
+  // instructions rather than generic ones
+  int n;
+  if (a.tables_in_smem && a.p2_in_smem) {
+    n = select_levels(a, sm, reinterpret_cast<const uint2*>(dyn), dyn + stage_off, tid);
+  } else {
+    unsigned char* const p2 = a.p2_in_smem
+                                  ? dyn + stage_off
+                                  : a.g_p2 + static_cast<size_t>(b) * a.p2_stride;
+    n = select_levels(a, sm, a.tables_in_smem ? reinterpret_cast<const uint2*>(dyn) : kids, p2,
+                      tid);
+  }
   if (tid == 0) a.n_nodes[b] = n;
   if (a.mask) {
     // the tree-attention mask and position ids (as presto_tree_mask computes them):

@@ -128,6 +128,17 @@ struct Elem<__nv_bfloat16> {
   }
 };
 
+// 16 bytes at a shared-memory address (an explicit shared load: a pointer computed
+// through integer arithmetic would otherwise be read with a generic one).
+__device__ __forceinline__ uint4 lds128(uint32_t saddr) {
+  uint4 r;
+  asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "r"(saddr)
+               : "memory");
+  return r;
+}
+
 __device__ __forceinline__ uint4 ldg_stream(const uint4* p) {
   uint4 r;
   asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
@@ -728,6 +739,7 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
       reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(dyn_raw) + 127) &
                                        ~static_cast<uintptr_t>(127)) +
       warp * kWStages * kWChunkBytes;
+  const uint32_t ring_s = smem_u32(ring);  // read with shared-memory loads, not generic ones
   if (lane == 0) {
     for (int s = 0; s < kWStages; ++s) mbar_init(&sh.full[warp][s], 1);
     sh.theta[warp] = -INFINITY;
@@ -819,8 +831,7 @@ __global__ void __launch_bounds__(kWThreads, 2) topk_stream_kernel(const Args a)
 #pragma unroll
     for (int i = 0; i < kWVec; ++i) {
       const int vi = i * 32 + lane;
-      d[i] = vi < nv ? *reinterpret_cast<const uint4*>(ring + sg * kWChunkBytes + vi * 16)
-                     : make_uint4(ni, ni, ni, ni);
+      d[i] = vi < nv ? lds128(ring_s + sg * kWChunkBytes + vi * 16) : make_uint4(ni, ni, ni, ni);
     }
     __syncwarp();
     if (lane == 0 && c + kWStages < nch) {  // the slot is free again: refill it

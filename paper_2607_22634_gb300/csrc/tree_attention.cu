@@ -622,7 +622,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int r0 = split * slice;
   const int nr = max(0, min(R, r0 + slice) - r0);
   // One item = one row of the slice x one column group (a bf16 quad or a float32
-  // pair), rows fastest (coalesced partial loads).  Each thread's first item is
+  // pair), rows fastest (coalesced partial loads).  Each thread's first two items are
   // loaded before the per-row weights are formed (one thread per row, into shared
   // memory), so the usual case costs one L2 round trip.
   auto merge = [&](auto wide_tag) {
@@ -638,8 +638,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         o[s] = (item < nitems && s < nsp) ? __ldcg(part + ((cta0 + s) * kCG + cg) * kBM + row)
                                          : PT{};
     };
-    PT oa[kMaxSplits];
+    PT oa[kMaxSplits], ob[kMaxSplits];
     load_item(tid, oa);
+    load_item(tid + kThreads, ob);
     if (tid < nr) {
       // the row's weights over the splits, w_s l_s / L (a split without keys for the
       // row has m = -inf and weight 0), and its lse
@@ -703,7 +704,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (cg == 0 && a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = mlse[i];
     };
     finish_item(tid, oa);
-    for (int item = tid + kThreads; item < nitems; item += kThreads) {
+    finish_item(tid + kThreads, ob);
+    for (int item = tid + 2 * kThreads; item < nitems; item += kThreads) {
       load_item(item, oa);
       finish_item(item, oa);
     }

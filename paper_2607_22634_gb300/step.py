@@ -140,6 +140,10 @@ class StagedRounds:
     two independent groups of requests, whose rounds do not wait on each other's
     results.  Every round still moves its own inputs in and its results out.
 
+    With a fixed pool of pinned host buffers (`fuse`), each round's step is one graph
+    replay: the round, the copy of its results out and, on a second stream beside it,
+    the copy of the next round's inputs in (`start_pooled`, `run_pooled`).
+
     `bind(views)` maps the staged tensors (a list of device views, in the order of
     `example`) to the arguments of DraftVerifyStep.run:
     (logits, ctx2, layers, kv_len, target_token).
@@ -159,6 +163,9 @@ class StagedRounds:
             for v, t in zip(self.views(buf), example):
                 v.copy_(t)
         self.graphs = [step.capture(*bind(self.views(s))) for s in self.staging]
+        self.bind = bind
+        self.pool = None  # pooled mode (fuse): data_ptr of a pool buffer -> its index
+        self.fused = {}
         self.copy_stream = torch.cuda.Stream(device=dev)
         self.result_host = [torch.empty(step.result.numel(), dtype=step.result.dtype).pin_memory()
                             for _ in range(2)]
@@ -208,3 +215,57 @@ class StagedRounds:
             self._launch(s ^ 1)
         self.read[s].synchronize()
         return self.result_host[s]
+
+    # ---- pooled mode: the host's inputs come from a fixed pool of pinned buffers
+    def fuse(self, host_bufs):
+        """Capture one CUDA graph per (pinned buffer j of a fixed pool, staging slot s): the
+        round on staging[s] and the copy of its results to result_host[s], and beside
+        them, on a second stream, the copy of pool buffer j into staging[s ^ 1] (the
+        inputs of the round after).  start_pooled() and run_pooled() then move one round
+        per graph replay, so the host's work per round is one replay and one wait."""
+        dev = self.step.device
+        cap = torch.cuda.Stream(device=dev)
+        self.pool = {hb.data_ptr(): j for j, hb in enumerate(host_bufs)}
+        cap.wait_stream(torch.cuda.current_stream(dev))
+        for j, hb in enumerate(host_bufs):
+            for s in (0, 1):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=cap):
+                    self.copy_stream.wait_stream(cap)
+                    with torch.cuda.stream(self.copy_stream):
+                        self.staging[s ^ 1].copy_(hb, non_blocking=True)
+                    self.step.run(*self.bind(self.views(self.staging[s])), stream=cap)
+                    self.result_host[s].copy_(self.step.result, non_blocking=True)
+                    cap.wait_stream(self.copy_stream)
+                self.fused[(j, s)] = g
+        torch.cuda.current_stream(dev).wait_stream(cap)
+
+    def _launch_pooled(self, s, after_next):
+        main = torch.cuda.current_stream(self.step.device)
+        if after_next is None:  # no round after this one: the round alone
+            self.graphs[s].replay()
+            self.result_host[s].copy_(self.step.result, non_blocking=True)
+        else:
+            self.fused[(self.pool[after_next.data_ptr()], s)].replay()
+        self.read[s].record(main)
+
+    def start_pooled(self, first, second=None):
+        """Queue round 0 (pool buffer `first`, copied in now) with round 1's inputs
+        (pool buffer `second`) copied in beside it."""
+        self.staging[0].copy_(first, non_blocking=True)
+        self._launch_pooled(0, second)
+
+    def run_pooled(self, i, after_next=None):
+        """Queue round i + 1 (its inputs were copied in beside round i) with pool buffer
+        `after_next` (round i + 2's inputs; None when round i + 1 is the last) copied in
+        beside it, then wait for round i and return its results on the host (rewritten
+        by round i + 2: copy them to keep them).  wait_pooled() collects the last round."""
+        s = i % 2
+        self._launch_pooled(s ^ 1, after_next)
+        self.read[s].synchronize()
+        return self.result_host[s]
+
+    def wait_pooled(self, i):
+        """Wait for round i, the last one queued, and return its results."""
+        self.read[i % 2].synchronize()
+        return self.result_host[i % 2]

@@ -1,6 +1,7 @@
 """StagedRounds (rounds fed from pinned host memory, one round queued ahead of the
-host): every round's returned accept results equal those of the same inputs run
-eagerly through DraftVerifyStep, across three rotating input sets."""
+host), both with separate copies and launches and in pooled mode (one captured graph
+per round step): every round's returned accept results equal those of the same
+inputs run eagerly through DraftVerifyStep, across three rotating input sets."""
 
 import numpy as np
 import torch
@@ -51,6 +52,17 @@ def test_staged_rounds_return_each_rounds_results():
     for i in range(n):
         got = staged.run(i, host[(i + 1) % 3] if i + 1 < n else None).numpy().copy()
         np.testing.assert_array_equal(got, want[i % 3], err_msg=f"round {i}")
+    torch.cuda.synchronize()
+    assert int(step.dev_status.item()) == 0
+    # pooled mode: one graph replay per round step
+    staged.fuse(host)
+    staged.start_pooled(host[0], host[1])
+    for i in range(n):
+        if i + 1 < n:
+            got = staged.run_pooled(i, host[(i + 2) % 3] if i + 2 < n else None)
+        else:
+            got = staged.wait_pooled(i)
+        np.testing.assert_array_equal(got.numpy().copy(), want[i % 3], err_msg=f"pooled round {i}")
     torch.cuda.synchronize()
     assert int(step.dev_status.item()) == 0
     # the sets really differ, so a round returning another round's results would fail

@@ -14,11 +14,12 @@
 //       - the elements >= tau (vectors whose maximum is below tau are skipped) become
 //         64-bit keys (value as an ordered integer, then the complement of the id,
 //         so "larger value, then lower id" is integer order) in a candidate buffer,
-//         ranked by counting.  If the buffer overflows (massive ties), an exact
-//         fallback raises a key threshold over the register-resident data until the
-//         survivors fit.
-//   * The leader CTA of the cluster merges the spans' (max, Σexp) pairs and top-k
-//     lists and writes the row.
+//         ranked by counting.  A span has few of them, so only the threads holding
+//         one work: one shared atomic each reserves their slots.  If the buffer
+//         overflows (massive ties), an exact fallback raises a key threshold over
+//         the register-resident data until the survivors fit.
+//   * The leader CTA of the cluster merges the spans' (max, Σexp) pairs (warp 0) and
+//     ranks their top-k lists (the other warps, at the same time), and writes the row.
 //   * With ENT the same pass also yields the row's entropy (App. F): next to
 //     s = Σ 2^u, u = x log2e - max2, each thread sums t = Σ 2^u u, and the merges
 //     carry t along (when the reference maximum drops by δ, t -> 2^δ (t + δ s)).
@@ -50,6 +51,8 @@ constexpr size_t kPrefetchCap = 48ull << 20;  // bytes a streaming launch asks L
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr unsigned kFull = 0xffffffffu;
 static_assert(kWarps >= kMaxK, "tau needs at least k warp maxima");
+static_assert(kWarps <= 32 && (kWarps & (kWarps - 1)) == 0, "the warp merge is a butterfly over kWarps lanes");
+static_assert(kMaxParts <= 32 && (kMaxParts & (kMaxParts - 1)) == 0, "the span merge is a butterfly over kMaxParts lanes");
 
 template <typename T>
 struct Elem;
@@ -250,7 +253,7 @@ __device__ __forceinline__ const T* row_base(const Args& a, int row, bool first)
 struct Smem {
   unsigned long long cand[kCandCap];
   unsigned long long list[kMaxK];               // the CTA's top-k, descending
-  unsigned long long part[kMaxParts][kMaxK];    // leader: the cluster's lists
+  unsigned long long part[kMaxParts * kMaxK];   // leader: the cluster's lists, span p at p * k
   float2 part_ms[kMaxParts];                    // leader: the cluster's (max, sum)
   float2 warp_ms[kWarps];                       // (max log2, sum) per warp
   float warp_t[kWarps];                         // ENT: entropy sum per warp
@@ -322,24 +325,26 @@ __device__ __forceinline__ void finish_row(const Args& a, SM& sh, int row, int p
   if (a.parts > 1) {
     cg::cluster_group cluster = cg::this_cluster();
     SM* leader = cluster.map_shared_rank(&sh, 0);
-    if (tid < k) leader->part[part][tid] = tid < got ? sh.list[tid] : 0ull;
+    if (tid < k) leader->part[part * k + tid] = tid < got ? sh.list[tid] : 0ull;
     if (tid == 0) {
       leader->part_ms[part] = make_float2(m_cta, s_cta);
       if constexpr (ENT) leader->part_t[part] = t_cta;
     }
     cluster.sync();
     if (part != 0) return;
-    // the parts' keys: zeros (fewer than k in a span) rank below every real key and
-    // are dropped below
+    // the leader: warps 1.. rank the spans' keys (zeros pad a span with fewer than k
+    // and rank below every real key), beside warp 0's merge of the spans' (max, sum)
     const int P = a.parts * k;
-    for (int i = tid; i < P; i += NT) sh.cand[i] = sh.part[i / k][i % k];
-    if (warp == 0) {
+    if (warp != 0) {
+      rank_keys<NT - 32>(sh.part, P, k, sh.list, tid - 32);
+    } else {
+      // lanes >= parts hold nothing: the butterfly stays within kMaxParts lanes
       float mw = lane < a.parts ? sh.part_ms[lane].x : -INFINITY;
       float sw = lane < a.parts ? sh.part_ms[lane].y : 0.f;
       float tw = 0.f;
       if constexpr (ENT) tw = lane < a.parts ? sh.part_t[lane] : 0.f;
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
+      for (int off = kMaxParts / 2; off > 0; off >>= 1) {
         const float m_o = __shfl_xor_sync(kFull, mw, off);
         const float s_o = __shfl_xor_sync(kFull, sw, off);
         if constexpr (ENT) {
@@ -349,12 +354,11 @@ __device__ __forceinline__ void finish_row(const Args& a, SM& sh, int row, int p
           merge_ms(mw, sw, m_o, s_o);
         }
       }
-      m_row = mw;
-      s_row = sw;
-      t_row = tw;
+      // write_row reads the pair in lanes 0..k-1
+      m_row = __shfl_sync(kFull, mw, 0);
+      s_row = __shfl_sync(kFull, sw, 0);
+      if constexpr (ENT) t_row = __shfl_sync(kFull, tw, 0);
     }
-    __syncthreads();
-    rank_keys<NT>(sh.cand, P, k, sh.list, tid);
     __syncthreads();
   }
   // ---- write the row (warp 0 holds the row's (max, sum))
@@ -500,88 +504,109 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
     hits |= (i < a.vpt && vi < v1 && E::vmax(d[i]) >= tau) ? (1u << i) : 0u;
   }
   const bool xhit = xid >= 0 && xval >= tau;
-  const uint32_t warp_hits = __reduce_or_sync(kFull, hits | (xhit ? 0x80000000u : 0u));
-  unsigned long long thr = 1ull;  // every real key is >= 1
-  int M;
-  for (;;) {
-    // count this thread's candidates, reserve their slots with one atomic per warp,
-    // then write them.  Vectors are visited under warp-uniform votes; a visited
-    // vector's elements >= tau form a bit mask from independent compares, and only
-    // those elements become keys
-    auto elem_mask = [&](int i) {
-      uint32_t em = 0u;
+  // the elements of vector i that are >= tau, as a bit mask from independent compares
+  auto ge_tau = [&](int i) {
+    uint32_t em = 0u;
 #pragma unroll
-      for (int e = 0; e < n; ++e) em |= (E::value(d[i], e) >= tau) ? (1u << e) : 0u;
-      return ((hits >> i) & 1u) ? em : 0u;
-    };
-    auto visit = [&](auto&& emit) {
+    for (int e = 0; e < n; ++e) em |= (E::value(d[i], e) >= tau) ? (1u << e) : 0u;
+    return em;
+  };
+  // every element >= tau becomes a candidate key.  Only the threads holding one (a
+  // few per span) do any work: each counts its elements, reserves their slots with
+  // one shared atomic and writes their keys
+  if (hits | static_cast<uint32_t>(xhit)) {
+    int mine = xhit ? 1 : 0;
 #pragma unroll
-      for (int i = 0; i < VMAX; ++i) {
-        if ((warp_hits >> i) & 1u) {  // warp-uniform
-          uint32_t em = elem_mask(i);
-          const int id0 = head + (v0 + i * kThreads + tid) * n;
-          while (em) {
-            const int e = __ffs(em) - 1;
-            em &= em - 1u;
-            const unsigned long long key = elem_key(E::value(d[i], e), id0 + e);
-            emit(key >= thr, key);
-          }
+    for (int i = 0; i < VMAX; ++i)
+      if ((hits >> i) & 1u) mine += __popc(ge_tau(i));
+    int slot = atomicAdd(&sh.count, mine);
+#pragma unroll
+    for (int i = 0; i < VMAX; ++i) {
+      if ((hits >> i) & 1u) {
+        uint32_t em = ge_tau(i);
+        const int id0 = head + (v0 + i * kThreads + tid) * n;
+        while (em) {
+          const int e = __ffs(em) - 1;
+          em &= em - 1u;
+          if (slot < kCandCap) sh.cand[slot] = elem_key(E::value(d[i], e), id0 + e);
+          ++slot;
         }
       }
-      if (warp_hits >> 31) {
-        const unsigned long long key = elem_key(xval, xid);
-        emit(xhit && key >= thr, key);
-      }
-    };
-    int mine = 0;
-    if (warp_hits && thr == 1ull) {  // every key passes: count the mask bits
-#pragma unroll
-      for (int i = 0; i < VMAX; ++i)
-        if ((warp_hits >> i) & 1u) mine += __popc(elem_mask(i));
-      mine += xhit;
-    } else if (warp_hits) {
-      visit([&](bool take, unsigned long long) { mine += take; });
     }
-    int incl = mine;  // inclusive prefix over the warp
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const int y = __shfl_up_sync(kFull, incl, off);
-      if (lane >= off) incl += y;
-    }
-    int base = 0;
-    if (lane == 31 && incl > 0) base = atomicAdd(&sh.count, incl);
-    base = __shfl_sync(kFull, base, 31) + incl - mine;
-    if (warp_hits)
-      visit([&](bool take, unsigned long long key) {
-        if (take && base < kCandCap) sh.cand[base] = key;
-        base += take;
-      });
-    __syncthreads();
-    M = sh.count;
-    if (M <= kCandCap) break;
-    // overflow: the k-th largest of the collected keys is <= the span's k-th largest
-    // key, so raising the threshold to it keeps the span's top-k; keys are unique, so
-    // it rises strictly and the rounds end
-    rank_keys(sh.cand, kCandCap, k, sh.list, tid);
-    __syncthreads();
-    if (tid == 0) {
-      sh.thr = sh.list[k - 1];
-      sh.count = 0;
-    }
-    __syncthreads();
-    thr = sh.thr;
+    if (xhit && slot < kCandCap) sh.cand[slot] = elem_key(xval, xid);
   }
-  // ---- the span's top-k
-  rank_keys(sh.cand, M, k, sh.list, tid);
-  // the span's (max, sum) from the warps'
+  __syncthreads();
+  int M = sh.count;
+  if (M > kCandCap) {
+    // overflow (massive ties; uniform across the CTA): the k-th largest of the keys
+    // collected is <= the span's k-th largest key, so the keys below it can go.  The
+    // rounds below collect the keys >= a threshold thr and raise it the same way
+    // until they fit; keys are unique, so it rises strictly and the rounds end
+    const uint32_t warp_hits = __reduce_or_sync(kFull, hits | (xhit ? 0x80000000u : 0u));
+    unsigned long long thr = 0ull;
+    for (;;) {
+      rank_keys(sh.cand, kCandCap, k, sh.list, tid);
+      __syncthreads();
+      if (tid == 0) {
+        sh.thr = sh.list[k - 1];
+        sh.count = 0;
+      }
+      __syncthreads();
+      thr = sh.thr;
+      // count this thread's keys >= thr, reserve their slots with one atomic per
+      // warp, then write them; vectors are visited under warp-uniform votes
+      auto visit = [&](auto&& emit) {
+#pragma unroll
+        for (int i = 0; i < VMAX; ++i) {
+          if ((warp_hits >> i) & 1u) {  // warp-uniform
+            uint32_t em = ((hits >> i) & 1u) ? ge_tau(i) : 0u;
+            const int id0 = head + (v0 + i * kThreads + tid) * n;
+            while (em) {
+              const int e = __ffs(em) - 1;
+              em &= em - 1u;
+              const unsigned long long key = elem_key(E::value(d[i], e), id0 + e);
+              emit(key >= thr, key);
+            }
+          }
+        }
+        if (warp_hits >> 31) {
+          const unsigned long long key = elem_key(xval, xid);
+          emit(xhit && key >= thr, key);
+        }
+      };
+      int mine = 0;
+      if (warp_hits) visit([&](bool take, unsigned long long) { mine += take; });
+      int incl = mine;  // inclusive prefix over the warp
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(kFull, incl, off);
+        if (lane >= off) incl += y;
+      }
+      int base = 0;
+      if (lane == 31 && incl > 0) base = atomicAdd(&sh.count, incl);
+      base = __shfl_sync(kFull, base, 31) + incl - mine;
+      if (warp_hits)
+        visit([&](bool take, unsigned long long key) {
+          if (take && base < kCandCap) sh.cand[base] = key;
+          base += take;
+        });
+      __syncthreads();
+      M = sh.count;
+      if (M <= kCandCap) break;
+    }
+  }
+  // ---- the span's top-k (warps 1..), beside warp 0's merge of the warps' (max, sum)
+  if (warp != 0) rank_keys<kThreads - 32>(sh.cand, M, k, sh.list, tid - 32);
   float m_cta = -INFINITY, s_cta = 0.f, t_cta = 0.f;
   if (warp == 0) {
     float mw = lane < kWarps ? sh.warp_ms[lane].x : -INFINITY;
     float sw = lane < kWarps ? sh.warp_ms[lane].y : 0.f;
     float tw = 0.f;
     if constexpr (ENT) tw = lane < kWarps ? sh.warp_t[lane] : 0.f;
+    // lanes >= kWarps hold nothing: merging them changes no bit, so the butterfly
+    // stays within the first kWarps lanes
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
+    for (int off = kWarps / 2; off > 0; off >>= 1) {
       const float m_o = __shfl_xor_sync(kFull, mw, off);
       const float s_o = __shfl_xor_sync(kFull, sw, off);
       if constexpr (ENT) {
@@ -591,6 +616,7 @@ __global__ void __launch_bounds__(kThreads, VMAX <= 4 ? 2 : 1) topk_kernel(const
         merge_ms(mw, sw, m_o, s_o);
       }
     }
+    // lanes 0..kWarps-1 hold the span's pair (write_row reads it in lanes 0..k-1)
     m_cta = mw;
     s_cta = sw;
     t_cta = tw;

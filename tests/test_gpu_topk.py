@@ -72,6 +72,23 @@ def test_topk_many_ties_and_masked_vocab():
     assert _check(x, 16) == 0
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_topk_candidate_overflow_in_register_kernel(dtype):
+    """Few rows (the register-resident kernel) whose spans hold far more elements at
+    or above the threshold than the candidate buffer: constant rows, two-valued rows
+    and a row whose top values repeat; the threshold is raised over the kept data
+    until the keys fit, and ties go to the lower id."""
+    g = torch.Generator().manual_seed(21)
+    V = 151936
+    x = torch.randn(1, 4, V, generator=g)
+    x[0, 0] = 1.25                                                  # constant
+    x[0, 1] = (torch.rand(V, generator=g) < 0.5).float()            # two values
+    x[0, 2, ::7] = 9.0                                              # repeated maximum
+    x[0, 3, 100000:] = 5.0                                          # tied tail
+    assert _check(x.to(dtype), 8) == 0
+    assert _check(x[:, :2, :20000].contiguous().to(dtype), 16) == 0
+
+
 def test_topk_large_magnitudes():
     g = torch.Generator().manual_seed(4)
     x = torch.randn(1, 4, 30000, generator=g) * 40

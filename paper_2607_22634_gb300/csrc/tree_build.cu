@@ -2,7 +2,10 @@
 // and best-first tree construction (§4.2, Alg. 2; a node is committed when it is
 // popped), plus the device-side trigram table (presto_ngram3_*).
 //
-// One thread-block cluster of 8 CTAs per sequence:
+// One thread-block cluster per sequence: 16 CTAs when every cluster of the launch fits
+// on the device at once, else 8 (the trigram probes of phase 1 are bound by the
+// issue of their scattered loads, one L1 wavefront per lane, so they spread over as
+// many SMs as the launch can hold):
 //   phase 1 (all CTAs): each CTA takes a share of the context pairs reachable in
 //     the candidate tree and computes, for every candidate j of depth d+1 under
 //     that context, s = log q + lambda log rho (hash-table probes, batched so their
@@ -105,6 +108,7 @@ struct Args {
   int use_table;
   int L, k, bf, N;
   int nctx_all;      // contexts of one sequence over all depths
+  int csize;         // CTAs of a sequence's cluster
   int per_cta;       // contexts each CTA of the cluster scores
   int tables_in_smem;
   unsigned char* g_tables;  // [B][tables_bytes] when the tables do not fit in smem
@@ -192,7 +196,8 @@ __device__ __forceinline__ void decode_ctx(int g, int k, int use_table, int& d, 
   }
 }
 constexpr size_t kDynSmemBudget = 200 * 1024;
-constexpr int kCluster = 8;
+constexpr int kCluster = 8;       // CTAs of a sequence's cluster (portable size) ...
+constexpr int kClusterWide = 16;  // ... or, when every cluster of a launch fits at once, this
 
 // Phase-2 scratch of the leader CTA (aliases the phase-1 staging area).  The kept
 // set A (non-root nodes, sorted by key, so A[r] is node r + 1) and the candidate
@@ -545,7 +550,7 @@ __device__ __forceinline__ int select_levels(const Args& a, Smem& sm, const uint
   // ---- write the tree: node 0 is the root, node r + 1 is A[r] for r + 1 < head, then
   // the tail rows
   for (int i = tid; i < N; i += kThreads) {
-    const size_t o = static_cast<size_t>(blockIdx.x / kCluster) * N + i;
+    const size_t o = static_cast<size_t>(blockIdx.x / a.csize) * N + i;
     uint64_t ke = 0ull;
     int pid = -1;
     if (i > 0 && i < head) {
@@ -588,7 +593,7 @@ __global__ void __launch_bounds__(kThreads, 1) build_kernel(const Args a) {
   __shared__ Smem sm;
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = static_cast<int>(cluster.block_rank());
-  const int b = blockIdx.x / kCluster;
+  const int b = blockIdx.x / a.csize;
   const int tid = threadIdx.x;
   const int L = a.L, k = a.k, nb = a.bf, use_table = a.use_table;
   const TableLayout tl(L, k, nb, use_table);
@@ -892,9 +897,9 @@ struct BuildPlan {
   size_t ws_tables;  // workspace bytes per sequence
   size_t ws_p2;
 };
-BuildPlan plan_build(int L, int k, int b, int N, int W, int use_table) {
+BuildPlan plan_build(int L, int k, int b, int N, int W, int use_table, int csize) {
   const TableLayout tl(L, k, b, use_table);
-  const int per = (contexts_all(L, k, use_table) + kCluster - 1) / kCluster;
+  const int per = (contexts_all(L, k, use_table) + csize - 1) / csize;
   const size_t st = align_up(static_cast<size_t>(per) * k * 4, 16);
   const size_t p2 = P2Layout(N, b, W).bytes;
   const size_t both = st > p2 ? st : p2;
@@ -917,13 +922,63 @@ BuildPlan plan_build(int L, int k, int b, int N, int W, int use_table) {
   }
   return pl;
 }
+
+// The kernel's attributes (the shared-memory budget, the wide cluster) and the number
+// of clusters of kClusterWide CTAs the device holds at once, set and queried once per
+// device; -1 when a call fails.
+int wide_clusters_resident() {
+  static PerDeviceOnce attrs;
+  static int resident[kMaxDevices];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return -1;
+  const cudaError_t e = attrs.run([dev] {
+    cudaError_t r = cudaFuncSetAttribute(build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(kDynSmemBudget));
+    if (r != cudaSuccess) return r;
+    resident[dev] = 0;
+    if (cudaFuncSetAttribute(build_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+        cudaSuccess) {
+      cudaGetLastError();  // no wide clusters on this device: the portable size only
+      return cudaSuccess;
+    }
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(kClusterWide);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kDynSmemBudget;  // the most a launch takes: one CTA per SM
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = kClusterWide;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, build_kernel, &cfg) != cudaSuccess) {
+      cudaGetLastError();
+      n = 0;
+    }
+    resident[dev] = n;
+    return cudaSuccess;
+  });
+  return e == cudaSuccess ? resident[dev] : -1;
+}
+
+// CTAs per sequence: the wide cluster when all B clusters of it are resident at once
+// (the phase-1 probes spread over twice the SMs), else the portable size; 0 on a
+// failed CUDA call.
+int build_cluster(int B) {
+  const int wide = wide_clusters_resident();
+  if (wide < 0) return 0;
+  return B <= wide ? kClusterWide : kCluster;
+}
 }  // namespace
 
 extern "C" size_t presto_build_workspace_ex(int B, int L, int k, int N, int beam_width) {
   if (B < 1 || L < 1 || k < 1 || N < 1 || beam_width < 1) return 0;
   // sized for the larger case (prefix signal, b = k): what any call with these
   // shapes keeps outside shared memory fits
-  const BuildPlan pl = plan_build(L, k, k, N, beam_width, 1);
+  // and for the portable cluster (each CTA's staging area is largest there)
+  const BuildPlan pl = plan_build(L, k, k, N, beam_width, 1, kCluster);
   if (pl.tables_in_smem && pl.p2_in_smem) return 256;
   const TableLayout tl(L, k, k, 1);
   return static_cast<size_t>(B) * (align_up(tl.bytes, 256) + align_up(P2Layout(N, k, beam_width).bytes, 256));
@@ -1020,8 +1075,11 @@ extern "C" int presto_score_build_tree_mask(
   a.bf = b;
   a.N = N;
   a.nctx_all = contexts_all(L, k, a.use_table);
-  a.per_cta = (a.nctx_all + kCluster - 1) / kCluster;
-  const BuildPlan pl = plan_build(L, k, b, N, beam_width, a.use_table);
+  const int csize = build_cluster(B);
+  if (csize < 1) return PRESTO_ERR_CUDA;
+  a.csize = csize;
+  a.per_cta = (a.nctx_all + csize - 1) / csize;
+  const BuildPlan pl = plan_build(L, k, b, N, beam_width, a.use_table, csize);
   a.tables_in_smem = pl.tables_in_smem;
   a.p2_in_smem = pl.p2_in_smem;
   const size_t need = static_cast<size_t>(B) * (pl.ws_tables + pl.ws_p2);
@@ -1043,20 +1101,14 @@ extern "C" int presto_score_build_tree_mask(
   a.dev_status = dev_status;
   const size_t smem = pl.smem;
   if (smem > kDynSmemBudget) return PRESTO_ERR_UNSUPPORTED;
-  static PerDeviceOnce smem_attr;
-  if (smem_attr.run([] {
-        return cudaFuncSetAttribute(build_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    static_cast<int>(kDynSmemBudget));
-      }) != cudaSuccess)
-    return PRESTO_ERR_CUDA;
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(static_cast<unsigned>(B) * kCluster);
+  cfg.gridDim = dim3(static_cast<unsigned>(B) * csize);
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kCluster;
+  attr[0].val.clusterDim.x = csize;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   attr[1] = pdl_attribute();
@@ -1122,7 +1174,9 @@ extern "C" int presto_score_build_tree_noalloc(
                                           policy, beam_width, N, node_token, node_parent,
                                           node_depth, node_score, n_nodes, kv_len, mask, pos_ids);
   if (arg_status != PRESTO_OK) return arg_status;
-  const BuildPlan pl = plan_build(L, k, b, N, beam_width, ngram != nullptr);
+  const int csize = build_cluster(B);
+  if (csize < 1) return PRESTO_ERR_CUDA;
+  const BuildPlan pl = plan_build(L, k, b, N, beam_width, ngram != nullptr, csize);
   const size_t need = static_cast<size_t>(B) * (pl.ws_tables + pl.ws_p2);
   if (need > kBuildStaticScratch) return PRESTO_ERR_UNSUPPORTED;
   void* ws = build_static_scratch();

@@ -1174,9 +1174,9 @@ extern "C" int presto_score_build_tree_noalloc(
                                           policy, beam_width, N, node_token, node_parent,
                                           node_depth, node_score, n_nodes, kv_len, mask, pos_ids);
   if (arg_status != PRESTO_OK) return arg_status;
-  const int csize = build_cluster(B);
-  if (csize < 1) return PRESTO_ERR_CUDA;
-  const BuildPlan pl = plan_build(L, k, b, N, beam_width, ngram != nullptr, csize);
+  // the plan of the portable cluster needs the most scratch of any cluster size (its
+  // staging areas are the largest), so this host-side check covers the launch's plan
+  const BuildPlan pl = plan_build(L, k, b, N, beam_width, ngram != nullptr, kCluster);
   const size_t need = static_cast<size_t>(B) * (pl.ws_tables + pl.ws_p2);
   if (need > kBuildStaticScratch) return PRESTO_ERR_UNSUPPORTED;
   void* ws = build_static_scratch();

@@ -74,7 +74,8 @@ struct Args {
   float scale_log2;
   __nv_bfloat16* out;
   float* lse;
-  float2* part_o;   // KV splits: O / l of each row, [CTA][column group][kBM]
+  float2* part_o;   // KV splits: O / l of each row, [CTA][column group][kBM] (groups of
+                    // 8 bf16 or, wide partials, 2 float32 columns)
   float2* part_ml;  // KV splits: (m, l) per row [CTA][kBM], log2 domain
   int32_t* dev_status;
 };
@@ -492,9 +493,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (ok) {
         tc_fence_after();
         // the row normalised by its own l (values stay within the range of V), laid
-        // out so that a warp's 32 rows of one column group are 256 contiguous bytes:
-        // bf16 column quads, or float32 column pairs when the sequence's prefix is
-        // short (wide partials)
+        // out so that a warp's 32 rows of one column group are contiguous: bf16
+        // column octets (512 bytes), or float32 column pairs (256 bytes) when the
+        // sequence's prefix is short (wide partials)
         const float inv = l > 0.f ? 1.f / l : 0.f;
 #pragma unroll 1
         for (int cc = 0; cc < D / 64; ++cc) {
@@ -509,14 +510,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int q = 0; q < 16; ++q)
               dst[(c * 16 + q) * kBM] = make_float2(o[q * 2] * inv, o[q * 2 + 1] * inv);
           } else {
-            uint2* dst = reinterpret_cast<uint2*>(a.part_o) +
-                         static_cast<size_t>(blockIdx.x) * (D / 4) * kBM + r;
+            uint4* dst = reinterpret_cast<uint4*>(a.part_o) +
+                         static_cast<size_t>(blockIdx.x) * (D / 8) * kBM + r;
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              const __nv_bfloat162 lo = __floats2bfloat162_rn(o[q * 4] * inv, o[q * 4 + 1] * inv);
-              const __nv_bfloat162 hi = __floats2bfloat162_rn(o[q * 4 + 2] * inv, o[q * 4 + 3] * inv);
-              dst[(c * 8 + q) * kBM] = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
-                                                  *reinterpret_cast<const uint32_t*>(&hi));
+            for (int q = 0; q < 4; ++q) {
+              uint4 w4;
+              uint32_t* w = reinterpret_cast<uint32_t*>(&w4);
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const __nv_bfloat162 o2 =
+                    __floats2bfloat162_rn(o[q * 8 + 2 * e] * inv, o[q * 8 + 2 * e + 1] * inv);
+                w[e] = *reinterpret_cast<const uint32_t*>(&o2);
+              }
+              dst[(c * 4 + q) * kBM] = w4;
             }
           }
         }
@@ -621,14 +627,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   const size_t cta0 = static_cast<size_t>(blockIdx.x - split);  // first CTA of the cluster
   const int r0 = split * slice;
   const int nr = max(0, min(R, r0 + slice) - r0);
-  // One item = one row of the slice x one column group (a bf16 quad or a float32
-  // pair), rows fastest (coalesced partial loads).  Each thread's first two items are
+  // One item = one row of the slice x one column group (a bf16 octet or a float32
+  // pair), rows fastest (coalesced partial loads).  Each thread's first items are
   // loaded before the per-row weights are formed (one thread per row, into shared
   // memory), so the usual case costs one L2 round trip.
   auto merge = [&](auto wide_tag) {
     constexpr bool kWide = decltype(wide_tag)::value;
-    using PT = std::conditional_t<kWide, float2, uint2>;
-    constexpr int kCG = kWide ? D / 2 : D / 4;  // column groups per row
+    using PT = std::conditional_t<kWide, float2, uint4>;
+    constexpr int kCG = kWide ? D / 2 : D / 8;  // column groups per row
     const PT* part = reinterpret_cast<const PT*>(a.part_o);
     const int nitems = nr * kCG;
     auto load_item = [&](int item, PT (&o)[kMaxSplits]) {
@@ -638,9 +644,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         o[s] = (item < nitems && s < nsp) ? __ldcg(part + ((cta0 + s) * kCG + cg) * kBM + row)
                                          : PT{};
     };
+    // items loaded before the weights: two of the float32 pairs, one of the bf16
+    // octets (a slice of kBM / 6 rows has about one octet item per thread)
+    constexpr int kAhead = kWide ? 2 : 1;
     PT oa[kMaxSplits], ob[kMaxSplits];
     load_item(tid, oa);
-    load_item(tid + kThreads, ob);
+    if constexpr (kAhead > 1) load_item(tid + kThreads, ob);
     if (tid < nr) {
       // the row's weights over the splits, w_s l_s / L (a split without keys for the
       // row has m = -inf and weight 0), and its lse
@@ -674,7 +683,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int node = mt * nodes_per_tile + row / a.G;
       const int hh = row % a.G;
       if (node >= a.N) return;
-      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int s = 0; s < kMaxSplits; ++s) {
         // weight 0: an absent split, or one without keys for this row (an empty
@@ -685,27 +694,33 @@ __global__ void __launch_bounds__(kThreads, 1)
             acc[0] = fmaf(w, o[s].x, acc[0]);
             acc[1] = fmaf(w, o[s].y, acc[1]);
           } else {
-            acc[0] = fmaf(w, __uint_as_float(o[s].x << 16), acc[0]);
-            acc[1] = fmaf(w, __uint_as_float(o[s].x & 0xffff0000u), acc[1]);
-            acc[2] = fmaf(w, __uint_as_float(o[s].y << 16), acc[2]);
-            acc[3] = fmaf(w, __uint_as_float(o[s].y & 0xffff0000u), acc[3]);
+            const uint32_t ow[4] = {o[s].x, o[s].y, o[s].z, o[s].w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              acc[2 * e] = fmaf(w, __uint_as_float(ow[e] << 16), acc[2 * e]);
+              acc[2 * e + 1] = fmaf(w, __uint_as_float(ow[e] & 0xffff0000u), acc[2 * e + 1]);
+            }
           }
         }
       }
       const size_t orow = ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
-      const __nv_bfloat162 lo = __floats2bfloat162_rn(acc[0], acc[1]);
       if constexpr (kWide) {
-        *reinterpret_cast<__nv_bfloat162*>(a.out + orow + cg * 2) = lo;
+        *reinterpret_cast<__nv_bfloat162*>(a.out + orow + cg * 2) = __floats2bfloat162_rn(acc[0], acc[1]);
       } else {
-        const __nv_bfloat162 hi = __floats2bfloat162_rn(acc[2], acc[3]);
-        *reinterpret_cast<uint2*>(a.out + orow + cg * 4) =
-            make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+        uint4 w4;
+        uint32_t* w = reinterpret_cast<uint32_t*>(&w4);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const __nv_bfloat162 o2 = __floats2bfloat162_rn(acc[2 * e], acc[2 * e + 1]);
+          w[e] = *reinterpret_cast<const uint32_t*>(&o2);
+        }
+        *reinterpret_cast<uint4*>(a.out + orow + cg * 8) = w4;
       }
       if (cg == 0 && a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = mlse[i];
     };
     finish_item(tid, oa);
-    finish_item(tid + kThreads, ob);
-    for (int item = tid + 2 * kThreads; item < nitems; item += kThreads) {
+    if constexpr (kAhead > 1) finish_item(tid + kThreads, ob);
+    for (int item = tid + kAhead * kThreads; item < nitems; item += kThreads) {
       load_item(item, oa);
       finish_item(item, oa);
     }

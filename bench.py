@@ -780,11 +780,12 @@ def time_full_depth(args, P):
               for q in range(w.B))
     kvh = kv.cpu().numpy()
     flops = 4.0 * w.Hq * w.D * (sum(int(kvh[q]) * int(n_nodes[q]) for q in range(w.B)) + anc)
+    launches = step.kernels_per_round(w.layers)
     del layers, step, g
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
     return {"workload": "long_ctx: B=8 L=16 k=10 N=256 T=32768, 36 attention layers",
-            "ms_per_round": ms, "rounds_per_s": 1e3 / ms, "gpu_launches_per_round": 3 + w.layers,
+            "ms_per_round": ms, "rounds_per_s": 1e3 / ms, "gpu_launches_per_round": launches,
             "attention_tflops": flops * w.layers / (ms * 1e-3) / 1e12,
             "kv_cache_gb": kv_bytes / 1e9}
 
@@ -1064,7 +1065,8 @@ def run_ours(args):
         else:
             ach = attn_bytes / (t_us * 1e-6) / 1e9
             roof = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s"}
-        roof["kernel"] = "presto_tree_attention (attn_kernel)"
+        roof["kernel"] = ("presto_tree_attention (attn_kernel" +
+                          (" + attn_merge_kernel)" if step.attn_launches > 1 else ")"))
         roof["traffic"] = profiled_traffic("attention")
         roof["tensor_frac"] = attn_flops / (t_us * 1e-6) / 1e12 / tc
         roof["tensor_frac_sustained"] = attn_flops / (t_us * 1e-6) / 1e12 / tc_sus

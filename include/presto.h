@@ -393,6 +393,10 @@ int presto_tree_mask(const int32_t* node_parent, const int32_t* node_depth,
  * q, k_tree, v_tree, mask and n_nodes are read after that wait.
  */
 size_t presto_attn_workspace(int B, int N, int Hq, int Hkv, int D, int Tmax);
+/* Kernels one presto_tree_attention call of these shapes launches on the current
+ * device: 2 when its KV splits are merged by a second kernel, else 1; 0 for shapes
+ * the call refuses (the checks of presto_attn_workspace). */
+int presto_attn_launches(int B, int N, int Hq, int Hkv, int D, int Tmax);
 int presto_tree_attention(const void* q, const void* k_cache, const void* v_cache,
                           const int32_t* kv_len, int Tmax, const void* k_tree,
                           const void* v_tree, const uint32_t* mask, const int32_t* n_nodes,

@@ -20,6 +20,7 @@ from ._lib import (  # noqa: F401
     load,
     pack_trigram_keys,
     presto_accept,
+    presto_attn_launches,
     presto_attn_workspace,
     presto_build_flags,
     presto_build_workspace,

@@ -70,6 +70,7 @@ _SIGS = {
                                      ctypes.c_size_t, _P, _P]),
     "presto_tree_mask": (_I, [_P, _P, _P, _P, _I, _I, _P, _P, _P, _P]),
     "presto_attn_workspace": (ctypes.c_size_t, [_I, _I, _I, _I, _I, _I]),
+    "presto_attn_launches": (_I, [_I, _I, _I, _I, _I, _I]),
     "presto_tree_attention": (_I, [_P, _P, _P, _P, _I, _P, _P, _P, _P, _I, _I, _I, _I, _I,
                                    ctypes.c_float, _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "presto_accept": (_I, [_P, _P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P]),
@@ -408,6 +409,11 @@ def presto_tree_mask(node_parent, node_depth, n_nodes, kv_len, mask=None, pos_id
 
 def presto_attn_workspace(B, N, Hq, Hkv, D, Tmax) -> int:
     return int(load().presto_attn_workspace(B, N, Hq, Hkv, D, Tmax))
+
+
+def presto_attn_launches(B, N, Hq, Hkv, D, Tmax) -> int:
+    """Kernels one presto_tree_attention call of these shapes launches (0: refused)."""
+    return int(load().presto_attn_launches(B, N, Hq, Hkv, D, Tmax))
 
 
 def presto_tree_attention(q, k_cache, v_cache, kv_len, k_tree, v_tree, mask, n_nodes,

@@ -25,17 +25,18 @@
 //     rescaled in TMEM, after the previous PV completed) when it grows by more than
 //     2^8, so most tiles skip the rescale;
 //   * with several KV splits (a row tile's prefix and tree-key tiles dealt out in
-//     equal runs), the splits of one row tile form a thread-block cluster (up to 16
-//     CTAs): each CTA writes its rows' fp32 (m, l) and O / l to the workspace (bf16
-//     column quads, or float32 column pairs when the prefix is short; coalesced
-//     either way), the cluster synchronises (release / acquire), and each CTA
-//     merges a slice of the rows over the splits with log-sum-exp weights, all loads
-//     of a row issued together.
+//     equal runs; the split count fills the SMs, up to 16), each CTA writes its
+//     rows' fp32 (m, l) and O / l to the workspace (bf16 column octets, or float32
+//     column pairs when the prefix is short; coalesced either way) and exits.  A
+//     second kernel, launched behind it on the stream (programmatic dependent
+//     launch: its CTAs start early and wait for the first grid's results), merges
+//     the rows over the splits with log-sum-exp weights, 16 rows of a row tile per
+//     CTA and all loads of a row issued together.  Splits that are plain CTAs, not
+//     a cluster, are not limited by how many clusters of their size fit at once.
 // Every wait is bounded; on time-out the CTA records PRESTO_DEV_TIMEOUT, lets its
 // copies and MMAs in flight complete (bounded), then frees its TMEM and exits.
 #include <cuda_bf16.h>
 
-#include <cooperative_groups.h>
 #include <cudaTypedefs.h>
 
 #include <cmath>
@@ -131,7 +132,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kc,
                 const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ CUtensorMap tm_kt,
                 const __grid_constant__ CUtensorMap tm_vt, const Args a) {
-  namespace cg = cooperative_groups;
   using Ly = Layout<D>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -141,8 +141,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ int abort_flag;
   __shared__ float xmax[2][2][kBM];  // per iteration parity and half: the half-row maxima
   __shared__ float xl[2][kBM];       // per half: the half-row sums
-  __shared__ float mw[kBM][kMaxSplits + 1];  // split merge: per-row weights (slice <= kBM rows)
-  __shared__ float mlse[kBM];                // split merge: per-row lse
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   int idx = blockIdx.x;
@@ -152,7 +150,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   idx /= a.n_mt;
   const int g = idx % a.Hkv;
   const int b = idx / a.Hkv;
-  const bool clustered = a.n_splits > 1;
+  const bool partial = a.n_splits > 1;  // KV splits: this CTA leaves a partial result
   const int nodes_per_tile = kBM / a.G;
   pdl_launch_dependents();
 
@@ -485,7 +483,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __all_sync(0xffffffffu, mbar_wait(&bars.o_done, (nt - 1) & 1, abort));
       if (!ok) fail();
     }
-    if (clustered) {
+    if (partial) {
       // this split's normalised row and (m, l) for the merge (a failed or empty row
       // is marked by m = -inf and contributes nothing); each half writes its columns
       const size_t prow = static_cast<size_t>(blockIdx.x) * kBM + r;
@@ -585,48 +583,63 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
 
-  if (!clustered) {
-    if (nt == 0 && tid < kBM) {  // no keys at all: a zero row, lse -inf
-      const int r = tid;
-      const int node = mt * nodes_per_tile + r / a.G, hh = r % a.G;
-      if (node < a.N) {
-        __nv_bfloat16* orow =
-            a.out + ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
-        for (int c = 0; c < D; c += 8) *reinterpret_cast<uint4*>(orow + c) = make_uint4(0, 0, 0, 0);
-        if (a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = -INFINITY;
-      }
+  if (partial) {
+    if (nt == 0 && tid < kBM)  // an empty split contributes nothing
+      a.part_ml[static_cast<size_t>(blockIdx.x) * kBM + tid] = make_float2(-INFINITY, 0.f);
+  } else if (nt == 0 && tid < kBM) {  // no keys at all: a zero row, lse -inf
+    const int r = tid;
+    const int node = mt * nodes_per_tile + r / a.G, hh = r % a.G;
+    if (node < a.N) {
+      __nv_bfloat16* orow =
+          a.out + ((static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh) * D;
+      for (int c = 0; c < D; c += 8) *reinterpret_cast<uint4*>(orow + c) = make_uint4(0, 0, 0, 0);
+      if (a.lse) a.lse[(static_cast<size_t>(b) * a.N + node) * a.Hq + g * a.G + hh] = -INFINITY;
     }
-    tc_fence_before();
-    __syncthreads();
-    if (warp == kMmaWarp) {
-      tc_fence_after();
-      tmem_dealloc(tmem_base, kTmemCols);
-    }
-    return;
   }
-
-  // ---------------------------------------------------------------- split merge
-  // The KV splits of this row tile are the CTAs of the cluster; each has left its
-  // rows' (m, l) and normalised O in the workspace.  Rows are dealt out in slices,
-  // one per CTA, and each CTA combines its slice over the splits with log-sum-exp
-  // weights (the partials stay in L2).
-  if (nt == 0 && tid < kBM)  // an empty split contributes nothing
-    a.part_ml[static_cast<size_t>(blockIdx.x) * kBM + tid] = make_float2(-INFINITY, 0.f);
   tc_fence_before();
   __syncthreads();
   if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem_base, kTmemCols);
   }
-  // release / acquire at cluster scope: every split's partial rows are visible
-  cg::this_cluster().sync();
+}
+
+// ---------------------------------------------------------------- split merge
+// One CTA per kMergeRows rows of a row tile: the KV splits of the row tile (CTAs
+// cta0 .. cta0 + n_splits - 1 of attn_kernel) have left each row's (m, l) and
+// normalised O in the workspace, and the rows are combined with log-sum-exp weights
+// (the partials stay in L2).  Launched right behind attn_kernel with programmatic
+// dependent launch: the CTAs may start while it runs and wait for its results.
+constexpr int kMergeRows = 16;
+constexpr int kMergeThreads = 256;
+static_assert(kBM % kMergeRows == 0, "a row tile is whole merge slices");
+
+template <int D>
+__global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const Args a) {
+  __shared__ float mw[kMergeRows][kMaxSplits + 1];  // per-row weights over the splits
+  __shared__ float mlse[kMergeRows];                // per-row lse
+  constexpr int kThreads = kMergeThreads;  // the merge body's block size
+  constexpr int kSlices = kBM / kMergeRows;
+  const int tid = threadIdx.x;
+  int idx = blockIdx.x;
+  const int slice = idx % kSlices;
+  idx /= kSlices;
+  const int mt = idx % a.n_mt;
+  idx /= a.n_mt;
+  const int g = idx % a.Hkv;
+  const int b = idx / a.Hkv;
+  const int nodes_per_tile = kBM / a.G;
+  pdl_launch_dependents();
+  pdl_wait();  // the partials come from attn_kernel
+  // the partials' precision, as attn_kernel chose it (which reports a bad kv_len)
+  int kv = ld_chain(a.kv_len + b);
+  kv = kv < 0 ? 0 : (kv > a.Tmax ? a.Tmax : kv);
+  const bool wide = kv < kWidePartialKeys;
   const int nn = min(max(ld_chain(a.n_nodes + b), 0), a.N);
-  const int R = kBM;
   const int nsp = a.n_splits;
-  const int slice = (R + nsp - 1) / nsp;
-  const size_t cta0 = static_cast<size_t>(blockIdx.x - split);  // first CTA of the cluster
-  const int r0 = split * slice;
-  const int nr = max(0, min(R, r0 + slice) - r0);
+  const size_t cta0 = ((static_cast<size_t>(b) * a.Hkv + g) * a.n_mt + mt) * nsp;
+  const int r0 = slice * kMergeRows;
+  const int nr = kMergeRows;
   // One item = one row of the slice x one column group (a bf16 octet or a float32
   // pair), rows fastest (coalesced partial loads).  Each thread's first items are
   // loaded before the per-row weights are formed (one thread per row, into shared
@@ -645,7 +658,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                          : PT{};
     };
     // items loaded before the weights: two of the float32 pairs, one of the bf16
-    // octets (a slice of kBM / 6 rows has about one octet item per thread)
+    // octets (a slice has one octet item per thread at D = 128)
     constexpr int kAhead = kWide ? 2 : 1;
     PT oa[kMaxSplits], ob[kMaxSplits];
     load_item(tid, oa);
@@ -738,25 +751,26 @@ struct Plan {
   size_t ctas;
 };
 
-// active[s] = how many clusters of s CTAs (s = 1..kMaxSplits) can be resident on
-// the GPU at once; 0 where that cluster size does not fit.
-Plan make_plan(int B, int N, int Hq, int Hkv, int Tmax, const int* active) {
+// resident = how many CTAs of the kernel the GPU holds at once.
+Plan make_plan(int B, int N, int Hq, int Hkv, int Tmax, int resident) {
   Plan p;
   p.G = Hq / Hkv;
   p.n_mt = (N * p.G + kBM - 1) / kBM;
   const int tiles = (Tmax + kBN - 1) / kBN + (N + kBN - 1) / kBN;
   int max_splits = tiles / 2 > 1 ? tiles / 2 : 1;
   if (max_splits > kMaxSplits) max_splits = kMaxSplits;
-  // The split count by the estimated time: waves of resident clusters x (KV tiles of
-  // the busiest CTA -- the tiles are dealt out in runs of ceil(tiles / s) -- plus a
-  // fixed cost of about three tiles), lightly penalising splits (each adds rows to
-  // merge), so that of two split counts with the same runs the smaller wins.
+  // The split count by the estimated time: waves of resident row tiles (each s
+  // CTAs) x (KV tiles of the busiest CTA -- the tiles are dealt out in runs of
+  // ceil(tiles / s) -- plus a fixed cost of about three tiles), lightly penalising
+  // splits (each adds rows to merge), so that of two split counts with the same runs
+  // the smaller wins.
   const long long units = static_cast<long long>(B) * Hkv * p.n_mt;
   double best_cost = 1e30;
   p.n_splits = 1;
   for (int s = 1; s <= max_splits; ++s) {
-    if (active[s] < 1) continue;
-    const double waves = std::ceil(static_cast<double>(units) / active[s]);
+    const int active = resident / s;
+    if (active < 1) continue;
+    const double waves = std::ceil(static_cast<double>(units) / active);
     const int run = (tiles + s - 1) / s;
     const double cost = waves * (run + 3.0) * (1.0 + 0.02 * (s - 1));
     if (cost < best_cost - 1e-9) {
@@ -768,56 +782,37 @@ Plan make_plan(int B, int N, int Hq, int Hkv, int Tmax, const int* active) {
   return p;
 }
 
-// The kernel's shared-memory limit and its permission for clusters of more than 8
-// CTAs, set once on every device that launches it.
+// The kernel's shared-memory limit, set once on every device that launches it.
 template <int D>
 cudaError_t set_smem_attr() {
   static PerDeviceOnce attr;
   return attr.run([] {
-    cudaError_t e = cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         Layout<D>::kAlloc);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    return e;
+    return cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                Layout<D>::kAlloc);
   });
 }
 
-// Resident-cluster counts for cluster sizes 1..kMaxSplits, for this kernel's block
-// size and shared memory (queried once per device and D).
+// CTAs of the kernel resident on the GPU at once (queried once per device and D;
+// one SM's worth if the query fails).
 template <int D>
-const int* active_clusters() {
-  static int cached[64][kMaxSplits + 1];
-  static bool done[64] = {false};
+int resident_ctas() {
+  static int cached[kMaxDevices];
+  static bool done[kMaxDevices] = {false};
   static std::mutex mu;
   int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) dev = 0;
   std::lock_guard<std::mutex> lock(mu);
-  int* act = cached[dev];
-  if (done[dev]) return act;
-  if (set_smem_attr<D>() != cudaSuccess) cudaGetLastError();
-  act[0] = 0;
-  for (int c = 1; c <= kMaxSplits; ++c) {
-    cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3(c);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = Layout<D>::kAlloc;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = c;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, attn_kernel<D>, &cfg) != cudaSuccess) {
-      cudaGetLastError();
-      n = 0;
-    }
-    act[c] = n;
+  if (done[dev]) return cached[dev];
+  int per_sm = 0;
+  if (set_smem_attr<D>() != cudaSuccess ||
+      cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, attn_kernel<D>, kThreads,
+                                                    Layout<D>::kAlloc) != cudaSuccess) {
+    cudaGetLastError();
+    per_sm = 0;
   }
-  if (act[1] < 1) act[1] = sm_count();  // a lone CTA always fits
+  cached[dev] = per_sm > 0 ? per_sm * sm_count() : 1;
   done[dev] = true;
-  return act;
+  return cached[dev];
 }
 
 }  // namespace
@@ -850,10 +845,18 @@ extern "C" size_t presto_attn_workspace(int B, int N, int Hq, int Hkv, int D, in
     return 0;
   if (use_pair(B, N, Hq, Hkv, D, Tmax)) return pair_attn::workspace(B, N, Hq, Hkv, D, Tmax);
   // KV splits leave partial rows (float32 at most) and fp32 (m, l) for the merge
-  const int* active = D == 128 ? active_clusters<128>() : active_clusters<64>();
-  const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
+  const int resident = D == 128 ? resident_ctas<128>() : resident_ctas<64>();
+  const Plan p = make_plan(B, N, Hq, Hkv, Tmax, resident);
   if (p.n_splits == 1) return 256;
   return align_up(p.ctas * kBM * (static_cast<size_t>(D) * 4 + 8), 256);
+}
+
+extern "C" int presto_attn_launches(int B, int N, int Hq, int Hkv, int D, int Tmax) {
+  if (B < 1 || N < 1 || Hq < 1 || Hkv < 1 || Hq % Hkv || Tmax < 1 || (D != 64 && D != 128))
+    return 0;
+  if (use_pair(B, N, Hq, Hkv, D, Tmax)) return 1;
+  const int resident = D == 128 ? resident_ctas<128>() : resident_ctas<64>();
+  return make_plan(B, N, Hq, Hkv, Tmax, resident).n_splits > 1 ? 2 : 1;
 }
 
 extern "C" int presto_tree_attention(const void* q, const void* k_cache, const void* v_cache,
@@ -876,8 +879,8 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
   if (use_pair(B, N, Hq, Hkv, D, Tmax))
     return pair_attn::launch(q, k_cache, v_cache, kv_len, Tmax, k_tree, v_tree, mask, n_nodes, B, N,
                              Hq, Hkv, D, sm_scale, out, lse, ws, ws_bytes, dev_status, stream);
-  const int* active = D == 128 ? active_clusters<128>() : active_clusters<64>();
-  const Plan p = make_plan(B, N, Hq, Hkv, Tmax, active);
+  const int resident = D == 128 ? resident_ctas<128>() : resident_ctas<64>();
+  const Plan p = make_plan(B, N, Hq, Hkv, Tmax, resident);
   Args a{};
   if (p.n_splits > 1) {
     const size_t need = p.ctas * kBM * (static_cast<size_t>(D) * 4 + 8);
@@ -921,14 +924,10 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
   cfg.gridDim = dim3(static_cast<unsigned>(p.ctas));
   cfg.blockDim = dim3(kThreads);
   cfg.stream = stream;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = p.n_splits;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  attr[1] = pdl_attribute();
+  cudaLaunchAttribute attr[1];
+  attr[0] = pdl_attribute();
   cfg.attrs = attr;
-  cfg.numAttrs = 2;
+  cfg.numAttrs = 1;
   cudaError_t err;
   if (D == 128) {
     if (set_smem_attr<128>() != cudaSuccess) return PRESTO_ERR_CUDA;
@@ -940,6 +939,17 @@ extern "C" int presto_tree_attention(const void* q, const void* k_cache, const v
     err = cudaLaunchKernelEx(&cfg, attn_kernel<64>, tq, tkc, tvc, tkt, tvt, a);
   }
   if (err != cudaSuccess) return PRESTO_ERR_CUDA;
+  if (p.n_splits > 1) {  // the merge of the splits, right behind on the stream
+    cudaLaunchConfig_t mc{};
+    mc.gridDim = dim3(static_cast<unsigned>(p.ctas / p.n_splits) * (kBM / kMergeRows));
+    mc.blockDim = dim3(kMergeThreads);
+    mc.stream = stream;
+    mc.attrs = attr;
+    mc.numAttrs = 1;
+    err = D == 128 ? cudaLaunchKernelEx(&mc, attn_merge_kernel<128>, a)
+                   : cudaLaunchKernelEx(&mc, attn_merge_kernel<64>, a);
+    if (err != cudaSuccess) return PRESTO_ERR_CUDA;
+  }
   return launch_status();
 }
 

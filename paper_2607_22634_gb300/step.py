@@ -53,6 +53,7 @@ class DraftVerifyStep:
         self.ws_build = torch.empty(max(P.presto_build_workspace(B, L, k, N), 1), dtype=u8, device=dev)
         self.ws_attn = torch.empty(max(P.presto_attn_workspace(B, N, Hq, Hkv, D, Tmax), 1),
                                    dtype=u8, device=dev)
+        self.attn_launches = P.presto_attn_launches(B, N, Hq, Hkv, D, Tmax)
         self.graph = None
         self.fuse_mask = fuse_mask
         self.CALLS = (("topk", "build", "attention", "accept") if fuse_mask
@@ -109,9 +110,9 @@ class DraftVerifyStep:
 
     def kernels_per_round(self, n_layers=1):
         """Library kernels one round launches: top-k, tree build (with the mask when
-        fused, else a mask kernel too), accept and one attention kernel per layer (KV
-        splits merge inside the kernel)."""
-        return (3 if self.fuse_mask else 4) + n_layers
+        fused, else a mask kernel too), accept and, per layer, the attention kernels
+        (one, or two when a second kernel merges the KV splits)."""
+        return (3 if self.fuse_mask else 4) + n_layers * self.attn_launches
 
     def capture(self, logits, ctx2, layers, kv_len, target_token):
         """Capture one round on these exact input tensors into a CUDA graph."""

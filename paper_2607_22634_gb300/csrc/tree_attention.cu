@@ -630,11 +630,13 @@ __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const Args a)
   const int b = idx / a.Hkv;
   const int nodes_per_tile = kBM / a.G;
   pdl_launch_dependents();
-  pdl_wait();  // the partials come from attn_kernel
-  // the partials' precision, as attn_kernel chose it (which reports a bad kv_len)
+  // the partials' precision, as attn_kernel chose it (which reports a bad kv_len);
+  // no kernel of a round writes kv_len, so it is read before the dependency wait and
+  // the partial loads after it are the merge's only round trip
   int kv = ld_chain(a.kv_len + b);
   kv = kv < 0 ? 0 : (kv > a.Tmax ? a.Tmax : kv);
   const bool wide = kv < kWidePartialKeys;
+  pdl_wait();  // the partials come from attn_kernel (and the node count from the build)
   const int nn = min(max(ld_chain(a.n_nodes + b), 0), a.N);
   const int nsp = a.n_splits;
   const size_t cta0 = ((static_cast<size_t>(b) * a.Hkv + g) * a.n_mt + mt) * nsp;

@@ -610,7 +610,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // normalised O in the workspace, and the rows are combined with log-sum-exp weights
 // (the partials stay in L2).  Launched right behind attn_kernel with programmatic
 // dependent launch: the CTAs may start while it runs and wait for its results.
-constexpr int kMergeRows = 16;
+constexpr int kMergeRows = 8;
 constexpr int kMergeThreads = 256;
 static_assert(kBM % kMergeRows == 0, "a row tile is whole merge slices");
 

@@ -30,7 +30,7 @@
 //     column pairs when the prefix is short; coalesced either way) and exits.  A
 //     second kernel, launched behind it on the stream (programmatic dependent
 //     launch: its CTAs start early and wait for the first grid's results), merges
-//     the rows over the splits with log-sum-exp weights, 16 rows of a row tile per
+//     the rows over the splits with log-sum-exp weights, 8 rows of a row tile per
 //     CTA and all loads of a row issued together.  Splits that are plain CTAs, not
 //     a cluster, are not limited by how many clusters of their size fit at once.
 // Every wait is bounded; on time-out the CTA records PRESTO_DEV_TIMEOUT, lets its
@@ -660,7 +660,7 @@ __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const Args a)
                                          : PT{};
     };
     // items loaded before the weights: two of the float32 pairs, one of the bf16
-    // octets (a slice has one octet item per thread at D = 128)
+    // octets (a slice has at most one octet item per thread at D = 128)
     constexpr int kAhead = kWide ? 2 : 1;
     PT oa[kMaxSplits], ob[kMaxSplits];
     load_item(tid, oa);

@@ -366,31 +366,50 @@ __device__ __forceinline__ int select_levels(const Args& a, Smem& sm, const uint
         if (r == cap - 1) sm.tau = e < na ? akey[cur * N + e] : C[e - na];  // the new A's last key
       }
     } else {
-      for (int e = tid; e < ne; e += kThreads) {
-        int r;
-        if (e < na) {
-          const uint64_t ke = akey[cur * N + e];
-          r = e;
-          for (int i = 0; i < m; ++i) r += C[i] > ke;
-        } else {
-          const int ci = e - na;
-          const uint64_t ke = C[ci];
-          int lo = 0, hi = na;  // A entries with key >= ke
-          while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (akey[cur * N + mid] >= ke) lo = mid + 1;
-            else hi = mid;
+      // each entry's count of candidates above it is split over a group of G lanes
+      // (candidates g, g + G, ...; G a power of two, as many as the block holds) and
+      // summed across the group, so no thread runs a chain of m compares
+      int G = 1;
+      while (G < 32 && ne * (2 * G) <= kThreads) G *= 2;
+      const int total = ne * G;
+      for (int base = tid & ~31; base < total; base += kThreads) {  // warp-uniform
+        const int idx = base + lane;
+        const bool act = idx < total;
+        const int e = idx / G, g = idx & (G - 1);
+        uint64_t ke = 0ull;
+        int ci = -1;  // a candidate's own index (ties to the lower index); -1 for A entries
+        if (act) {
+          if (e < na) {
+            ke = akey[cur * N + e];
+          } else {
+            ci = e - na;
+            ke = C[ci];
           }
-          int rc = 0;
-          for (int i = 0; i < m; ++i) {
-            const uint64_t ki = C[i];
-            rc += ki > ke || (ki == ke && i < ci);
-          }
-          rkc[ci] = static_cast<int16_t>(rc);
-          r = lo + rc;
         }
-        rk[e] = static_cast<int16_t>(r < cap ? r : cap);
-        if (r == cap - 1) sm.tau = e < na ? akey[cur * N + e] : C[e - na];  // the new A's last key
+        int cnt = 0;
+        if (act)
+          for (int i = g; i < m; i += G) {
+            const uint64_t ki = C[i];
+            cnt += ki > ke || (ki == ke && i < ci);
+          }
+        for (int off = G >> 1; off > 0; off >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, off);
+        if (act && g == 0) {
+          int r;
+          if (e < na) {
+            r = e + cnt;
+          } else {
+            int lo = 0, hi = na;  // A entries with key >= ke
+            while (lo < hi) {
+              const int mid = (lo + hi) >> 1;
+              if (akey[cur * N + mid] >= ke) lo = mid + 1;
+              else hi = mid;
+            }
+            rkc[ci] = static_cast<int16_t>(cnt);
+            r = lo + cnt;
+          }
+          rk[e] = static_cast<int16_t>(r < cap ? r : cap);
+          if (r == cap - 1) sm.tau = ke;  // the new A's last key
+        }
       }
     }
     if (tid == 0) sm.nc[cc ^ 1] = 0;  // the next level's counter (last read a level ago)

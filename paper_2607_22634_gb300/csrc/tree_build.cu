@@ -230,6 +230,7 @@ struct P2Layout {
 };
 constexpr uint32_t kNoCtx = 0xFFFFFFFFu;
 constexpr int kSortMin = 256;  // candidates of a level above which they are sorted first
+static_assert(kSortMin < (1 << 16) && kMaxN < (1 << 15), "two counts share one int in the ranking");
 
 // Top-N selection of the candidate tree, level by level (leader CTA, all threads).
 //
@@ -386,26 +387,26 @@ __device__ __forceinline__ int select_levels(const Args& a, Smem& sm, const uint
             ke = C[ci];
           }
         }
+        // low half: candidates above the entry; high half (candidates only): entries of
+        // A with key >= ke, i.e. the candidate's position in the sorted A
         int cnt = 0;
-        if (act)
+        if (act) {
           for (int i = g; i < m; i += G) {
             const uint64_t ki = C[i];
             cnt += ki > ke || (ki == ke && i < ci);
           }
+          if (ci >= 0)
+            for (int i = g; i < na; i += G) cnt += (akey[cur * N + i] >= ke) << 16;
+        }
         for (int off = G >> 1; off > 0; off >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, off);
         if (act && g == 0) {
           int r;
+          const int rc = cnt & 0xFFFF;
           if (e < na) {
-            r = e + cnt;
+            r = e + rc;
           } else {
-            int lo = 0, hi = na;  // A entries with key >= ke
-            while (lo < hi) {
-              const int mid = (lo + hi) >> 1;
-              if (akey[cur * N + mid] >= ke) lo = mid + 1;
-              else hi = mid;
-            }
-            rkc[ci] = static_cast<int16_t>(cnt);
-            r = lo + cnt;
+            rkc[ci] = static_cast<int16_t>(rc);
+            r = (cnt >> 16) + rc;
           }
           rk[e] = static_cast<int16_t>(r < cap ? r : cap);
           if (r == cap - 1) sm.tau = ke;  // the new A's last key

@@ -19,7 +19,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr uint32_t kTmemCols = 512;
 constexpr int kWidePartialKeys = 1024;  // prefixes shorter than this merge float32 partials
-constexpr int kMaxSplits = 16;          // KV splits of a row block = CTAs of its cluster
+constexpr int kMaxSplits = 16;          // KV splits of a row block (long runs: the CTAs of its cluster)
 
 // Packed fp32 pairs (f32x2 arithmetic issues one instruction per two values) and
 // the three-input max.

@@ -125,6 +125,19 @@ def test_attention_qwen3_8b_round_full():
     _run_and_check(inp, t, w.N)
 
 
+def test_attention_launch_count():
+    """presto_attn_launches: the Qwen3-8B-shaped call splits its KV range over plain CTAs
+    and merges them in a second kernel; self_spec takes the long-run schedule (one
+    kernel, splits merged inside its clusters); refused shapes launch nothing."""
+    q = synth.WORKLOADS["qwen3_8b"]
+    assert P.presto_attn_launches(q.B, q.N, q.Hq, q.Hkv, q.D, q.T) == 2
+    s = synth.WORKLOADS["self_spec"]
+    assert P.presto_attn_launches(s.B, s.N, s.Hq, s.Hkv, s.D, s.T) == 1
+    assert P.presto_attn_launches(1, 8, 4, 1, 128, 16) == 1  # one KV tile: no split
+    assert P.presto_attn_launches(1, 8, 6, 4, 128, 16) == 0  # Hq not a multiple of Hkv
+    assert P.presto_attn_launches(1, 8, 4, 1, 96, 16) == 0   # unsupported D
+
+
 def test_attention_batched_ragged_sampled():
     w = synth.WORKLOADS["batched_ragged"]
     inp = synth.attention_inputs(w, device="cuda")

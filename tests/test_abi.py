@@ -98,6 +98,12 @@ def test_host_validation_rejects_bad_arguments():
     assert lib.presto_tree_attention(*att(128, 12, 4)) == -2      # G = 3 not a power of two
     assert lib.presto_tree_attention(*att(128, 8, 3)) == -1       # Hq % Hkv != 0
     assert lib.presto_tree_attention(*att(128, 8, 2, q=ctypes.c_void_p(24))) == -1
+    # attention queries: refused shapes size nothing and launch nothing (answered on the
+    # host, before any CUDA call)
+    for B, Nn, Hq, Hkv, D, T in ((0, 8, 8, 2, 128, 64), (1, 8, 8, 3, 128, 64),
+                                 (1, 8, 8, 2, 96, 64), (1, 8, 8, 2, 128, 0)):
+        assert lib.presto_attn_workspace(B, Nn, Hq, Hkv, D, T) == 0
+        assert lib.presto_attn_launches(B, Nn, Hq, Hkv, D, T) == 0
     # accept: L above limit
     assert lib.presto_accept(p, p, p, p, p, p, 1, 8, 64, p, p, p, N, N) == -2
     # table: capacity out of range
